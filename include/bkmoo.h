@@ -1,0 +1,212 @@
+/*
+ * bkmoo.h -- C ABI of the Bucket-Level MOO resolve library for GB300 (sm_103a).
+ *
+ * The method ("Multilingual Fine-Tuning via Localized Gradient Conflict
+ * Resolution", arXiv 2606.05613, Section 3.2 and Algorithm 1) splits the
+ * parameters into disjoint buckets and, for every bucket, resolves the K
+ * per-language gradients restricted to that bucket into one update
+ * direction with a multi-objective rule (MGDA, CAGrad or PCGrad).  The global
+ * update is the concatenation of the bucket directions (Section 3.2).
+ *
+ * Every rule needs the gradients only through the bucket's K x K Gram matrix
+ * G[i][j] = <g_i, g_j> (Eq. 3, Eq. 4, Eq. 5 are functions of inner products),
+ * and every rule's result is a linear combination d_b = sum_k beta_k g_k.  So
+ * one resolve is three device passes: Gram, per-bucket solve for beta, and
+ * combination.
+ *
+ * Notation: K = number of languages (the paper's T), B = number of buckets
+ * (the paper's K), N = elements per language gradient.
+ *
+ * Conventions common to every entry point:
+ *  - Every buffer is owned by the caller.  No entry point allocates device
+ *    memory; scratch lives in a caller-supplied workspace.
+ *  - Device work is asynchronous on the caller's `stream` (a cudaStream_t
+ *    passed as void*; NULL = the legacy default stream).  Argument errors are
+ *    returned synchronously; conditions found on the device are written to
+ *    per-bucket status words and to the workspace status word
+ *    (bkmoo_workspace_status).
+ *  - Gradients are K separate device buffers, each the flat per-language
+ *    gradient in the layout the plan describes, N elements, fp32 or bf16,
+ *    16-byte aligned.
+ *  - Offsets are int64 element offsets: offsets[0] = 0, strictly
+ *    increasing, offsets[B] = N.  Bucket b is [offsets[b], offsets[b+1]).
+ *  - 1 <= K <= 16.
+ */
+#ifndef BKMOO_H
+#define BKMOO_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Return codes and per-bucket status values. */
+typedef enum {
+  BKMOO_OK = 0,
+  BKMOO_ERR_INVALID = 1,          /* bad argument; nothing was launched    */
+  BKMOO_ERR_CUDA = 2,             /* a CUDA call failed                    */
+  BKMOO_ERR_NONFINITE = 3,        /* per bucket: Gram not finite, beta=1/K */
+  BKMOO_ERR_WORKSPACE = 4,        /* workspace not initialised for this
+                                     plan, or too small                    */
+  BKMOO_ERR_TIMEOUT = 5,          /* a bounded device wait gave up         */
+  BKMOO_ERR_BUFFER_TOO_SMALL = 6, /* an output array is too short          */
+  BKMOO_ERR_NOT_CONVERGED = 7     /* per bucket: the solver hit its
+                                     iteration cap without meeting the
+                                     stopping test; beta is the last
+                                     iterate                               */
+} bkmoo_status;
+
+/* The multi-objective rule applied to every bucket (Algorithm 1). */
+typedef enum {
+  BKMOO_MGDA = 0,   /* Eq. 3 / Eq. 6: min-norm point of the convex hull     */
+  BKMOO_PCGRAD = 1, /* Eq. 5 / Eq. 8: sequential projection of conflicts   */
+  BKMOO_CAGRAD = 2, /* Eq. 4 / Eq. 7: conflict-averse direction            */
+  BKMOO_MEAN = 3    /* the averaged gradient of plain fine-tuning          */
+} bkmoo_rule;
+
+typedef enum { BKMOO_F32 = 0, BKMOO_BF16 = 1 } bkmoo_dtype;
+
+/* bkmoo_params.flags */
+#define BKMOO_FLAG_CLOSED_FORM_K2 0x1u /* K = 2 MGDA by its closed form      */
+#define BKMOO_FLAG_POLISH 0x2u         /* exact active-set completion after
+                                          the Frank-Wolfe phase (MGDA and
+                                          CAGrad)                            */
+#define BKMOO_FLAG_FUSED 0x4u          /* one persistent launch that resolves
+                                          bucket after bucket while the
+                                          bucket is still in L2              */
+
+typedef struct {
+  int32_t max_iter; /* Frank-Wolfe iterations per bucket (MGDA, CAGrad)     */
+  double tol;       /* relative duality-gap stop of the Frank-Wolfe phase   */
+  double cagrad_c;  /* CAGrad c in [0, 1) (Eq. 4); the paper uses 0.5       */
+  uint64_t seed;    /* PCGrad "random order" (Algorithm 1) is a function of */
+  uint64_t step;    /*   (seed, step, bucket, task), see bkmoo_resolve      */
+  uint32_t flags;   /* BKMOO_FLAG_*                                         */
+} bkmoo_params;
+
+/* Fill *p with the defaults: max_iter 256, tol 1e-12, cagrad_c 0.5, seed 0,
+ * step 0, flags CLOSED_FORM_K2 | POLISH. */
+void bkmoo_default_params(bkmoo_params* p);
+
+/*
+ * bkmoo_plan -- bucket partition (Section 3.2, Figure 4 caption: fixed-size
+ * buckets filled during the backward pass starting from the last
+ * parameters).  Host only, pure.
+ *
+ * param_sizes[n_params]: element counts of the model's tensors in
+ * registration order.  The flat gradient the other calls read lists them in
+ * REVERSE registration order, each tensor in its own flat order.  A bucket
+ * holds at most cap = floor(bucket_bytes / elem_bytes) elements: a tensor
+ * that does not fit in the open bucket closes it; a tensor larger than cap is
+ * cut into cap-sized pieces; the rest joins the open bucket.  Empty tensors
+ * are skipped.
+ *
+ * Two-call use: with out_offsets == NULL only *n_buckets is set.  Otherwise
+ * out_offsets[0 .. *n_buckets] is written; out_cap is its length (>= B + 1,
+ * else BKMOO_ERR_BUFFER_TOO_SMALL).  BKMOO_ERR_INVALID on a NULL pointer,
+ * negative size, elem_bytes <= 0 or cap < 1.
+ */
+int bkmoo_plan(const int64_t* param_sizes, int32_t n_params, int32_t elem_bytes,
+               int64_t bucket_bytes, int64_t* out_offsets, int64_t out_cap,
+               int64_t* n_buckets);
+
+/*
+ * bkmoo_workspace_size -- bytes of device workspace that bkmoo_gram and
+ * bkmoo_resolve need for K languages of `in_dtype` over the buckets given by
+ * offsets[0 .. n_buckets] (host array).  Writes *bytes.  The workspace holds
+ * the device copy of the bucket table, per-block Gram partials (fp64), the
+ * per-bucket coefficients and a status word.
+ */
+int bkmoo_workspace_size(int32_t K, int32_t in_dtype, const int64_t* offsets,
+                         int64_t n_buckets, size_t* bytes);
+
+/*
+ * bkmoo_workspace_init -- write the bucket table for (K, in_dtype, offsets)
+ * into the workspace `ws` (device, ws_bytes >= bkmoo_workspace_size, 256-byte
+ * aligned).  Call once per plan and workspace, before the first bkmoo_gram or
+ * bkmoo_resolve with them.  Copies from host memory and synchronises
+ * `stream`.  Later calls must pass the same offsets: a different plan is
+ * detected on the device and reported as BKMOO_ERR_WORKSPACE.
+ */
+int bkmoo_workspace_init(int32_t K, int32_t in_dtype, const int64_t* offsets,
+                         int64_t n_buckets, void* ws, size_t ws_bytes,
+                         void* stream);
+
+/*
+ * bkmoo_gram -- per-bucket Gram matrices, the inner products every rule is
+ * built on (Eq. 2, the QP of Eq. 3 / Eq. 6 and the tests of Eq. 8 depend on
+ * the gradients only through them).
+ *
+ * grads: host array of K device pointers.  out_gram: device, fp64,
+ * [n_buckets][K][K], row-major, both triangles written.  Results are
+ * deterministic: each element is summed in fp32 within a thread over at most
+ * 128 elements, then reduced in a fixed order (warp tree in fp32, CTA and
+ * cross-CTA in fp64); no atomics.
+ */
+int bkmoo_gram(const void* const* grads, int32_t K, int32_t in_dtype,
+               const int64_t* offsets, int64_t n_buckets, double* out_gram,
+               void* ws, size_t ws_bytes, void* stream);
+
+/*
+ * bkmoo_resolve -- the resolve of Algorithm 1 for every bucket: Gram ->
+ * rule -> d_b = sum_k beta_k g_k, written into the flat direction out_dir
+ * (the concatenation of Section 3.2).
+ *
+ * grads / K / in_dtype / offsets / n_buckets as in bkmoo_gram.
+ * rule: bkmoo_rule.  p: parameters (NULL = defaults).
+ *  - MGDA: Frank-Wolfe on the simplex QP from the best pair (exact line
+ *    search, at most p->max_iter steps, stop at duality gap <= p->tol
+ *    relative to max_k G_kk), then, with BKMOO_FLAG_POLISH, an exact
+ *    active-set (Wolfe minimum-norm-point) completion.  K = 2 with
+ *    BKMOO_FLAG_CLOSED_FORM_K2 uses
+ *    gamma = clamp(<g2 - g1, g2> / ||g1 - g2||^2, 0, 1).  beta = alpha.
+ *  - CAGrad: the dual min_{w in simplex} <g0, g_w> + c ||g0|| ||g_w||
+ *    (g0 the mean) by Frank-Wolfe with exact line search, then the same
+ *    active-set completion; beta = 1/K + c ||g0|| w / ||g_w||.  No rescaling.
+ *  - PCGrad: for each task t, other tasks j in t's order, project the
+ *    running d_t off the ORIGINAL g_j when <d_t, g_j> < 0; d = sum_t d_t.
+ *    The order of task t in bucket b is a Fisher-Yates shuffle of the
+ *    ascending list [0..K-1] without t, slot i = m-1 .. 1 (m = K-1) swapped
+ *    with slot r mod (i+1), r the draws mix64(k3 + (n+1) * 0x9E3779B97F4A7C15)
+ *    for n = 0, 1, ..., where k1 = mix64(seed + (step+1) * G),
+ *    k2 = mix64(k1 + (b+1) * G), k3 = mix64(k2 + (t+1) * G),
+ *    G = 0x9E3779B97F4A7C15 and mix64 is the SplitMix64 output function.
+ *  - MEAN: beta = 1/K.
+ * out_dir: device, N elements of out_dtype (fp32 or bf16, round to nearest
+ *   even).  It may be exactly one of the grads buffers when the dtypes match
+ *   (in-place); any other overlap with a gradient is BKMOO_ERR_INVALID.
+ * out_weights: device fp32 [n_buckets][K] = beta, or NULL.
+ * out_status: device int32 [n_buckets] = BKMOO_OK, BKMOO_ERR_NONFINITE (the
+ *   Gram had a NaN/Inf; beta = 1/K), BKMOO_ERR_NOT_CONVERGED or
+ *   BKMOO_ERR_WORKSPACE; or NULL.
+ * ws / ws_bytes: the workspace after bkmoo_workspace_init with the same
+ *   K, in_dtype and offsets.
+ * Returns BKMOO_OK once the work is queued on `stream`.
+ */
+int bkmoo_resolve(const void* const* grads, int32_t K, int32_t in_dtype,
+                  const int64_t* offsets, int64_t n_buckets, int32_t rule,
+                  const bkmoo_params* p, void* out_dir, int32_t out_dtype,
+                  float* out_weights, int32_t* out_status, void* ws,
+                  size_t ws_bytes, void* stream);
+
+/*
+ * bkmoo_workspace_status -- synchronise `stream` and read the workspace
+ * status word: BKMOO_OK, or the first device-side error recorded since the
+ * last bkmoo_gram / bkmoo_resolve started (BKMOO_ERR_WORKSPACE,
+ * BKMOO_ERR_TIMEOUT).  Writes *status.
+ */
+int bkmoo_workspace_status(const void* ws, void* stream, int32_t* status);
+
+/* Static English text for a bkmoo_status value. */
+const char* bkmoo_status_string(int32_t status);
+
+/* Library version, major * 10000 + minor * 100 + patch. */
+int32_t bkmoo_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* BKMOO_H */
