@@ -84,10 +84,15 @@ typedef struct {
   uint64_t seed;    /* PCGrad "random order" (Algorithm 1) is a function of */
   uint64_t step;    /*   (seed, step, bucket, task), see bkmoo_resolve      */
   uint32_t flags;   /* BKMOO_FLAG_*                                         */
+  void* events;     /* tracing: NULL, or an array of 4 cudaEvent_t that
+                       bkmoo_resolve records on `stream` before the Gram pass,
+                       after it, after the solve and after the combination
+                       (one persistent launch: the middle two are recorded
+                       together after it).  Owned by the caller.           */
 } bkmoo_params;
 
 /* Fill *p with the defaults: max_iter 256, tol 1e-12, cagrad_c 0.5, seed 0,
- * step 0, flags CLOSED_FORM_K2 | POLISH. */
+ * step 0, flags CLOSED_FORM_K2 | POLISH, events NULL. */
 void bkmoo_default_params(bkmoo_params* p);
 
 /*

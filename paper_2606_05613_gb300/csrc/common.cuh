@@ -1,0 +1,189 @@
+// Internal definitions shared by the translation units of the bkmoo CUDA
+// library: workspace layout, kernel argument blocks, 16-byte vector access
+// and the chunk -> bucket lookup.  Not part of the C ABI (include/bkmoo.h).
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stddef.h>
+#include <stdint.h>
+
+#include "bkmoo.h"
+
+namespace bkmoo {
+
+constexpr int kMaxK = 16;
+constexpr int kThreads = 256;              // CTA size of the streaming kernels
+constexpr int kWarps = kThreads / 32;
+constexpr int kVecPerThread = 16;          // 16-byte vectors per thread per Gram chunk
+constexpr uint32_t kMagic = 0x4f4d4b42u;   // "BKMO"
+constexpr int kSolveWarpsPerBlock = 4;
+
+__host__ __device__ constexpr int tri(int K) { return K * (K + 1) / 2; }
+__host__ __device__ constexpr int elems_per_vec(int dtype) { return dtype == BKMOO_F32 ? 4 : 8; }
+__host__ __device__ constexpr int64_t chunk_elems(int dtype) {
+  return (int64_t)kThreads * kVecPerThread * elems_per_vec(dtype);
+}
+
+// First 256 bytes of every workspace.
+struct WsHeader {
+  uint32_t magic;
+  int32_t K;
+  int32_t in_dtype;
+  int32_t status;        // device-side error word: BKMOO_OK or the first error
+  int64_t n_buckets;
+  int64_t n_elems;
+  int64_t n_chunks;
+  int64_t chunk_elems;
+  uint64_t plan_hash;
+  int64_t reserved[25];
+};
+static_assert(sizeof(WsHeader) == 256, "header is one 256-byte block");
+
+// Byte offsets of the workspace regions (identical on host and device).
+struct WsLayout {
+  size_t offsets;        // int64 [B + 1]   bucket boundaries (elements)
+  size_t chunk_prefix;   // int64 [B + 1]   first Gram chunk of each bucket
+  size_t partials;       // double [n_chunks][P] per-chunk Gram partials
+  size_t beta;           // float [B][K]    coefficients of the last resolve
+  size_t total;
+};
+
+__host__ __device__ inline size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
+
+__host__ __device__ inline WsLayout ws_layout(int K, int64_t B, int64_t n_chunks) {
+  WsLayout L;
+  size_t at = sizeof(WsHeader);
+  L.offsets = at;
+  at = align256(at + sizeof(int64_t) * (size_t)(B + 1));
+  L.chunk_prefix = at;
+  at = align256(at + sizeof(int64_t) * (size_t)(B + 1));
+  L.partials = at;
+  at = align256(at + sizeof(double) * (size_t)n_chunks * (size_t)tri(K));
+  L.beta = at;
+  at = align256(at + sizeof(float) * (size_t)B * (size_t)K);
+  L.total = at;
+  return L;
+}
+
+struct GradPtrs {
+  const void* p[kMaxK];
+};
+
+// Everything a kernel needs to find its data.
+struct PlanView {
+  WsHeader* hdr;
+  const int64_t* offsets;
+  const int64_t* chunk_prefix;
+  double* partials;
+  float* beta;
+  int64_t n_buckets;
+  int64_t n_chunks;
+  int64_t chunk_elems;
+  uint64_t plan_hash;
+  int32_t K;
+  int32_t in_dtype;
+};
+
+struct SolveParams {
+  int32_t rule;
+  int32_t max_iter;
+  double tol;
+  double cagrad_c;
+  uint64_t seed;
+  uint64_t step;
+  uint32_t flags;
+};
+
+// ---------------------------------------------------------------------------
+// Device helpers
+// ---------------------------------------------------------------------------
+
+__device__ __forceinline__ bool header_ok(const PlanView& v) {
+  const WsHeader* h = v.hdr;
+  return h->magic == kMagic && h->plan_hash == v.plan_hash && h->K == v.K &&
+         h->in_dtype == v.in_dtype && h->n_buckets == v.n_buckets &&
+         h->n_chunks == v.n_chunks;
+}
+
+__device__ __forceinline__ void record_error(WsHeader* h, int code) {
+  atomicCAS(&h->status, 0, code);
+}
+
+// Bucket b with chunk_prefix[b] <= w < chunk_prefix[b+1]; `hint` is tried
+// first (chunks of one CTA increase monotonically).
+__device__ __forceinline__ int64_t find_bucket(const int64_t* cp, int64_t B, int64_t w,
+                                               int64_t hint) {
+  if (hint < B && cp[hint] <= w && w < cp[hint + 1]) return hint;
+  if (hint + 1 < B && cp[hint + 1] <= w && w < cp[hint + 2]) return hint + 1;
+  int64_t lo = 0, hi = B;
+  while (hi - lo > 1) {
+    int64_t mid = (lo + hi) >> 1;
+    if (cp[mid] <= w) lo = mid;
+    else hi = mid;
+  }
+  return lo;
+}
+
+// 16-byte loads.  `nc`: read-only path, no L1 allocation (streams that are
+// read once by this kernel).  `cs`: coherent, evict-first (combine, which
+// may write in place over one of the inputs).
+__device__ __forceinline__ uint4 ld16_nc(const void* p) {
+  uint4 r;
+  asm volatile("ld.global.nc.L1::no_allocate.v4.u32 {%0,%1,%2,%3}, [%4];"
+               : "=r"(r.x), "=r"(r.y), "=r"(r.z), "=r"(r.w)
+               : "l"(p));
+  return r;
+}
+__device__ __forceinline__ uint4 ld16_cs(const void* p) {
+  uint4 r;
+  asm volatile("ld.global.cs.v4.u32 {%0,%1,%2,%3}, [%4];"
+               : "=r"(r.x), "=r"(r.y), "=r"(r.z), "=r"(r.w)
+               : "l"(p));
+  return r;
+}
+__device__ __forceinline__ void st16_cs(void* p, uint4 v) {
+  asm volatile("st.global.cs.v4.u32 [%0], {%1,%2,%3,%4};" ::"l"(p), "r"(v.x), "r"(v.y),
+               "r"(v.z), "r"(v.w)
+               : "memory");
+}
+__device__ __forceinline__ void st8_cs(void* p, uint2 v) {
+  asm volatile("st.global.cs.v2.u32 [%0], {%1,%2};" ::"l"(p), "r"(v.x), "r"(v.y) : "memory");
+}
+
+__device__ __forceinline__ uint32_t word(const uint4& r, int i) {
+  return i == 0 ? r.x : i == 1 ? r.y : i == 2 ? r.z : r.w;
+}
+
+// Element e of a 16-byte vector as fp32 (bf16 widened exactly).
+template <int DT>
+__device__ __forceinline__ float vec_elem(const uint4& r, int e) {
+  if (DT == BKMOO_F32) return __uint_as_float(word(r, e));
+  const uint32_t w = word(r, e >> 1);
+  return (e & 1) ? __uint_as_float(w & 0xffff0000u) : __uint_as_float(w << 16);
+}
+
+template <int DT>
+__device__ __forceinline__ float load_scalar(const void* base, int64_t i) {
+  if (DT == BKMOO_F32) return static_cast<const float*>(base)[i];
+  const uint16_t h = static_cast<const uint16_t*>(base)[i];
+  return __uint_as_float((uint32_t)h << 16);
+}
+
+// ---------------------------------------------------------------------------
+// Kernel tables and launchers
+// ---------------------------------------------------------------------------
+
+// Gram-pass kernels, signature (GradPtrs, PlanView); gram_f32.cu / gram_bf16.cu.
+const void* gram_partials_fn_f32(int K);
+const void* gram_partials_fn_bf16(int K);
+
+// Combine kernels, signature (GradPtrs, PlanView, void* out); combine_*.cu.
+const void* combine_fn_f32(int K, int dtype_out);
+const void* combine_fn_bf16(int K, int dtype_out);
+
+// solve.cu
+cudaError_t launch_solve(const PlanView& v, const SolveParams& p, float* out_weights,
+                         int32_t* out_status, cudaStream_t s);
+cudaError_t launch_gram_finalize(const PlanView& v, double* out_gram, cudaStream_t s);
+
+}  // namespace bkmoo

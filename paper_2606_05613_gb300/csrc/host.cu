@@ -1,0 +1,334 @@
+// Host side of the C ABI (include/bkmoo.h): argument checks, the bucket plan,
+// the workspace image and the launch sequence Gram -> solve -> combine on the
+// caller's stream.  Nothing here allocates device memory.
+#include <cuda_runtime.h>
+
+#include <cstring>
+#include <map>
+#include <mutex>
+#include <utility>
+#include <vector>
+
+#include "common.cuh"
+
+using namespace bkmoo;
+
+namespace {
+
+constexpr int32_t kVersion = 100;  // 0.1.0
+
+bool offsets_ok(const int64_t* off, int64_t B) {
+  if (!off || B < 0 || off[0] != 0) return false;
+  for (int64_t b = 0; b < B; ++b)
+    if (off[b + 1] <= off[b]) return false;
+  return true;
+}
+
+int64_t count_chunks(const int64_t* off, int64_t B, int64_t ch) {
+  int64_t n = 0;
+  for (int64_t b = 0; b < B; ++b) n += (off[b + 1] - off[b] + ch - 1) / ch;
+  return n;
+}
+
+// FNV-1a over the 64-bit words that define a plan.
+uint64_t plan_hash(int32_t K, int32_t dt, const int64_t* off, int64_t B) {
+  uint64_t h = 0xcbf29ce484222325ull;
+  auto mix = [&h](uint64_t x) {
+    h ^= x;
+    h *= 0x100000001b3ull;
+  };
+  mix((uint64_t)K);
+  mix((uint64_t)dt);
+  mix((uint64_t)B);
+  for (int64_t b = 0; b <= B; ++b) mix((uint64_t)off[b]);
+  return h;
+}
+
+bool dtype_ok(int32_t dt) { return dt == BKMOO_F32 || dt == BKMOO_BF16; }
+int elem_bytes(int32_t dt) { return dt == BKMOO_F32 ? 4 : 2; }
+bool aligned(const void* p, uintptr_t a) { return ((uintptr_t)p & (a - 1)) == 0; }
+
+struct LaunchCache {
+  std::mutex mu;
+  std::map<int, int> sms;
+  std::map<std::pair<int, const void*>, int> occ;
+};
+LaunchCache& cache() {
+  static LaunchCache c;
+  return c;
+}
+
+// Resident CTAs of `fn` on the current device times its SM count.
+cudaError_t persistent_grid(const void* fn, int threads, int* grid) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  LaunchCache& c = cache();
+  std::lock_guard<std::mutex> lk(c.mu);
+  auto it = c.sms.find(dev);
+  if (it == c.sms.end()) {
+    int n = 0;
+    e = cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+    if (e != cudaSuccess) return e;
+    it = c.sms.emplace(dev, n).first;
+  }
+  auto key = std::make_pair(dev, fn);
+  auto jt = c.occ.find(key);
+  if (jt == c.occ.end()) {
+    int n = 0;
+    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, fn, threads, 0);
+    if (e != cudaSuccess) return e;
+    jt = c.occ.emplace(key, n < 1 ? 1 : n).first;
+  }
+  *grid = it->second * jt->second;
+  return cudaSuccess;
+}
+
+const void* gram_fn(int K, int dt) {
+  return dt == BKMOO_F32 ? gram_partials_fn_f32(K) : gram_partials_fn_bf16(K);
+}
+const void* combine_fn(int K, int dti, int dto) {
+  return dti == BKMOO_F32 ? combine_fn_f32(K, dto) : combine_fn_bf16(K, dto);
+}
+
+// Common checks of bkmoo_gram / bkmoo_resolve; fills the plan view.
+int prepare(const void* const* grads, int32_t K, int32_t dt, const int64_t* offsets,
+            int64_t B, void* ws, size_t ws_bytes, PlanView* v, GradPtrs* g) {
+  if (K < 1 || K > kMaxK || !dtype_ok(dt) || !grads || !ws) return BKMOO_ERR_INVALID;
+  if (!offsets_ok(offsets, B)) return BKMOO_ERR_INVALID;
+  if (!aligned(ws, 256)) return BKMOO_ERR_INVALID;
+  for (int k = 0; k < K; ++k)
+    if (!grads[k] || !aligned(grads[k], 16)) return BKMOO_ERR_INVALID;
+  const int64_t ch = chunk_elems(dt);
+  const int64_t nch = count_chunks(offsets, B, ch);
+  const WsLayout L = ws_layout(K, B, nch);
+  if (ws_bytes < L.total) return BKMOO_ERR_WORKSPACE;
+  char* base = static_cast<char*>(ws);
+  v->hdr = reinterpret_cast<WsHeader*>(base);
+  v->offsets = reinterpret_cast<const int64_t*>(base + L.offsets);
+  v->chunk_prefix = reinterpret_cast<const int64_t*>(base + L.chunk_prefix);
+  v->partials = reinterpret_cast<double*>(base + L.partials);
+  v->beta = reinterpret_cast<float*>(base + L.beta);
+  v->n_buckets = B;
+  v->n_chunks = nch;
+  v->chunk_elems = ch;
+  v->plan_hash = plan_hash(K, dt, offsets, B);
+  v->K = K;
+  v->in_dtype = dt;
+  std::memset(g, 0, sizeof(*g));
+  for (int k = 0; k < K; ++k) g->p[k] = grads[k];
+  return BKMOO_OK;
+}
+
+int launch_gram_pass(const GradPtrs& g, const PlanView& v, cudaStream_t s) {
+  if (cudaMemsetAsync(&v.hdr->status, 0, sizeof(int32_t), s) != cudaSuccess)
+    return BKMOO_ERR_CUDA;
+  if (v.n_chunks == 0) return BKMOO_OK;
+  const void* fn = gram_fn(v.K, v.in_dtype);
+  int grid = 0;
+  if (persistent_grid(fn, kThreads, &grid) != cudaSuccess) return BKMOO_ERR_CUDA;
+  if (grid > v.n_chunks) grid = (int)v.n_chunks;
+  GradPtrs ga = g;
+  PlanView va = v;
+  void* args[] = {&ga, &va};
+  if (cudaLaunchKernel(fn, dim3(grid), dim3(kThreads), args, 0, s) != cudaSuccess)
+    return BKMOO_ERR_CUDA;
+  return BKMOO_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+void bkmoo_default_params(bkmoo_params* p) {
+  if (!p) return;
+  p->max_iter = 256;
+  p->tol = 1e-12;
+  p->cagrad_c = 0.5;
+  p->seed = 0;
+  p->step = 0;
+  p->flags = BKMOO_FLAG_CLOSED_FORM_K2 | BKMOO_FLAG_POLISH;
+  p->events = nullptr;
+}
+
+int bkmoo_plan(const int64_t* param_sizes, int32_t n_params, int32_t elem_bytes_,
+               int64_t bucket_bytes, int64_t* out_offsets, int64_t out_cap,
+               int64_t* n_buckets) {
+  if (!n_buckets || n_params < 0 || (n_params > 0 && !param_sizes) || elem_bytes_ <= 0 ||
+      bucket_bytes <= 0)
+    return BKMOO_ERR_INVALID;
+  const int64_t cap = bucket_bytes / elem_bytes_;
+  if (cap < 1) return BKMOO_ERR_INVALID;
+  for (int32_t i = 0; i < n_params; ++i)
+    if (param_sizes[i] < 0) return BKMOO_ERR_INVALID;
+
+  // Walk the tensors last-registered first; `fill` is the open bucket's size
+  // and `end` the flat position reached so far.
+  std::vector<int64_t> bounds;
+  bounds.push_back(0);
+  int64_t fill = 0, end = 0;
+  for (int32_t i = n_params; i-- > 0;) {
+    int64_t left = param_sizes[i];
+    if (left == 0) continue;
+    if (fill > 0 && fill + left > cap) {  // does not fit: close the open bucket
+      bounds.push_back(end);
+      fill = 0;
+    }
+    while (left > cap) {  // oversize tensor: whole cap-sized pieces
+      end += cap;
+      bounds.push_back(end);
+      left -= cap;
+    }
+    fill += left;
+    end += left;
+  }
+  if (fill > 0) bounds.push_back(end);
+  *n_buckets = (int64_t)bounds.size() - 1;
+  if (!out_offsets) return BKMOO_OK;
+  if (out_cap < (int64_t)bounds.size()) return BKMOO_ERR_BUFFER_TOO_SMALL;
+  std::memcpy(out_offsets, bounds.data(), sizeof(int64_t) * bounds.size());
+  return BKMOO_OK;
+}
+
+int bkmoo_workspace_size(int32_t K, int32_t in_dtype, const int64_t* offsets,
+                         int64_t n_buckets, size_t* bytes) {
+  if (!bytes || K < 1 || K > kMaxK || !dtype_ok(in_dtype) || !offsets_ok(offsets, n_buckets))
+    return BKMOO_ERR_INVALID;
+  const int64_t nch = count_chunks(offsets, n_buckets, chunk_elems(in_dtype));
+  *bytes = ws_layout(K, n_buckets, nch).total;
+  return BKMOO_OK;
+}
+
+int bkmoo_workspace_init(int32_t K, int32_t in_dtype, const int64_t* offsets,
+                         int64_t n_buckets, void* ws, size_t ws_bytes, void* stream) {
+  if (K < 1 || K > kMaxK || !dtype_ok(in_dtype) || !ws || !aligned(ws, 256) ||
+      !offsets_ok(offsets, n_buckets))
+    return BKMOO_ERR_INVALID;
+  const int64_t ch = chunk_elems(in_dtype);
+  const int64_t nch = count_chunks(offsets, n_buckets, ch);
+  const WsLayout L = ws_layout(K, n_buckets, nch);
+  if (ws_bytes < L.total) return BKMOO_ERR_WORKSPACE;
+  // Host image of header + bucket table, copied in one transfer.
+  std::vector<unsigned char> img(L.partials, 0);
+  WsHeader h;
+  std::memset(&h, 0, sizeof h);
+  h.magic = kMagic;
+  h.K = K;
+  h.in_dtype = in_dtype;
+  h.status = BKMOO_OK;
+  h.n_buckets = n_buckets;
+  h.n_elems = offsets[n_buckets];
+  h.n_chunks = nch;
+  h.chunk_elems = ch;
+  h.plan_hash = plan_hash(K, in_dtype, offsets, n_buckets);
+  std::memcpy(img.data(), &h, sizeof h);
+  std::memcpy(img.data() + L.offsets, offsets, sizeof(int64_t) * (size_t)(n_buckets + 1));
+  int64_t* cp = reinterpret_cast<int64_t*>(img.data() + L.chunk_prefix);
+  cp[0] = 0;
+  for (int64_t b = 0; b < n_buckets; ++b) cp[b + 1] = cp[b] + (offsets[b + 1] - offsets[b] + ch - 1) / ch;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if (cudaMemcpyAsync(ws, img.data(), img.size(), cudaMemcpyHostToDevice, s) != cudaSuccess)
+    return BKMOO_ERR_CUDA;
+  if (cudaStreamSynchronize(s) != cudaSuccess) return BKMOO_ERR_CUDA;
+  return BKMOO_OK;
+}
+
+int bkmoo_gram(const void* const* grads, int32_t K, int32_t in_dtype, const int64_t* offsets,
+               int64_t n_buckets, double* out_gram, void* ws, size_t ws_bytes, void* stream) {
+  if (!out_gram && n_buckets > 0) return BKMOO_ERR_INVALID;
+  PlanView v;
+  GradPtrs g;
+  int r = prepare(grads, K, in_dtype, offsets, n_buckets, ws, ws_bytes, &v, &g);
+  if (r != BKMOO_OK) return r;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  r = launch_gram_pass(g, v, s);
+  if (r != BKMOO_OK) return r;
+  if (launch_gram_finalize(v, out_gram, s) != cudaSuccess) return BKMOO_ERR_CUDA;
+  return BKMOO_OK;
+}
+
+int bkmoo_resolve(const void* const* grads, int32_t K, int32_t in_dtype, const int64_t* offsets,
+                  int64_t n_buckets, int32_t rule, const bkmoo_params* p, void* out_dir,
+                  int32_t out_dtype, float* out_weights, int32_t* out_status, void* ws,
+                  size_t ws_bytes, void* stream) {
+  if (rule < BKMOO_MGDA || rule > BKMOO_MEAN || !dtype_ok(out_dtype)) return BKMOO_ERR_INVALID;
+  if (!out_dir || !aligned(out_dir, 16)) return BKMOO_ERR_INVALID;
+  bkmoo_params prm;
+  if (p) prm = *p;
+  else bkmoo_default_params(&prm);
+  if (prm.max_iter < 0 || !(prm.cagrad_c >= 0.0 && prm.cagrad_c < 1.0) || !(prm.tol >= 0.0))
+    return BKMOO_ERR_INVALID;
+  PlanView v;
+  GradPtrs g;
+  int r = prepare(grads, K, in_dtype, offsets, n_buckets, ws, ws_bytes, &v, &g);
+  if (r != BKMOO_OK) return r;
+  // out_dir may be exactly one gradient (same dtype); any other overlap is refused.
+  const uintptr_t N = (uintptr_t)offsets[n_buckets];
+  const uintptr_t o0 = (uintptr_t)out_dir, o1 = o0 + N * elem_bytes(out_dtype);
+  for (int k = 0; k < K; ++k) {
+    const uintptr_t g0 = (uintptr_t)grads[k], g1 = g0 + N * elem_bytes(in_dtype);
+    if (o0 < g1 && g0 < o1 && !(o0 == g0 && out_dtype == in_dtype)) return BKMOO_ERR_INVALID;
+  }
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  cudaEvent_t* ev = static_cast<cudaEvent_t*>(prm.events);
+  if (ev && cudaEventRecord(ev[0], s) != cudaSuccess) return BKMOO_ERR_CUDA;
+  r = launch_gram_pass(g, v, s);
+  if (r != BKMOO_OK) return r;
+  if (ev && cudaEventRecord(ev[1], s) != cudaSuccess) return BKMOO_ERR_CUDA;
+  SolveParams sp;
+  sp.rule = rule;
+  sp.max_iter = prm.max_iter;
+  sp.tol = prm.tol;
+  sp.cagrad_c = prm.cagrad_c;
+  sp.seed = prm.seed;
+  sp.step = prm.step;
+  sp.flags = prm.flags;
+  if (launch_solve(v, sp, out_weights, out_status, s) != cudaSuccess) return BKMOO_ERR_CUDA;
+  if (ev && cudaEventRecord(ev[2], s) != cudaSuccess) return BKMOO_ERR_CUDA;
+  if (v.n_chunks == 0) {
+    if (ev && cudaEventRecord(ev[3], s) != cudaSuccess) return BKMOO_ERR_CUDA;
+    return BKMOO_OK;
+  }
+  const void* fn = combine_fn(K, in_dtype, out_dtype);
+  int grid = 0;
+  if (persistent_grid(fn, kThreads, &grid) != cudaSuccess) return BKMOO_ERR_CUDA;
+  if (grid > v.n_chunks) grid = (int)v.n_chunks;
+  PlanView va = v;
+  GradPtrs ga = g;
+  void* outp = out_dir;
+  void* args[] = {&ga, &va, &outp};
+  if (cudaLaunchKernel(fn, dim3(grid), dim3(kThreads), args, 0, s) != cudaSuccess)
+    return BKMOO_ERR_CUDA;
+  if (ev && cudaEventRecord(ev[3], s) != cudaSuccess) return BKMOO_ERR_CUDA;
+  return BKMOO_OK;
+}
+
+int bkmoo_workspace_status(const void* ws, void* stream, int32_t* status) {
+  if (!ws || !status || !aligned(ws, 256)) return BKMOO_ERR_INVALID;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if (cudaStreamSynchronize(s) != cudaSuccess) return BKMOO_ERR_CUDA;
+  const WsHeader* h = static_cast<const WsHeader*>(ws);
+  int32_t st = 0;
+  if (cudaMemcpy(&st, &h->status, sizeof st, cudaMemcpyDeviceToHost) != cudaSuccess)
+    return BKMOO_ERR_CUDA;
+  *status = st;
+  return BKMOO_OK;
+}
+
+const char* bkmoo_status_string(int32_t status) {
+  switch (status) {
+    case BKMOO_OK: return "ok";
+    case BKMOO_ERR_INVALID: return "invalid argument";
+    case BKMOO_ERR_CUDA: return "CUDA error";
+    case BKMOO_ERR_NONFINITE: return "non-finite Gram matrix (beta = 1/K)";
+    case BKMOO_ERR_WORKSPACE: return "workspace too small or not initialised for this plan";
+    case BKMOO_ERR_TIMEOUT: return "bounded device wait timed out";
+    case BKMOO_ERR_BUFFER_TOO_SMALL: return "output buffer too small";
+    case BKMOO_ERR_NOT_CONVERGED: return "solver stopped at its iteration cap";
+    default: return "unknown status";
+  }
+}
+
+int32_t bkmoo_version(void) { return kVersion; }
+
+}  // extern "C"

@@ -138,6 +138,14 @@ def qwen3_8b() -> Workload:
                     conflict_frac=0.02, rho_conflict=-0.7, sigma_lognormal=True)
 
 
+def qwen3_8b_layers(n_layers: int) -> Workload:
+    """Qwen3-8B decoder-layer shapes only (no embedding / LM head), n_layers
+    layers: the same kernels as the full model on a few GB (profiling)."""
+    sizes = qwen3_8b_sizes()[1:1 + 11 * n_layers]
+    return dataclasses.replace(qwen3_8b(), name="qwen3-8b-%dlayers-k4-bf16" % n_layers,
+                               param_sizes=tuple(sizes))
+
+
 def sweep(K: int, bucket_mib: int, n: int = 1_000_000_000) -> Workload:
     """1e9-element fp32 vector, N(0,1) gradients with a shared part at rho=0.3."""
     return Workload(f"sweep-k{K}-{bucket_mib}mib-f32", K, "f32", (n,), bucket_mib * MiB,

@@ -1,0 +1,156 @@
+"""CPU-side checks of the C ABI: the library loads, exports every declared
+symbol, its host-only plan is bit-exact against the oracle, and argument
+errors are rejected synchronously (no GPU needed, no kernel launched)."""
+import ctypes
+import os
+import re
+
+import numpy as np
+import pytest
+
+from oracle import oracle as orc
+from paper_2606_05613_gb300 import build as nb
+from paper_2606_05613_gb300 import inputs
+from paper_2606_05613_gb300 import native as bk
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    nb.build()
+    bk.load()
+
+
+def _declared_symbols():
+    hdrs = [os.path.join(ROOT, "include", f) for f in os.listdir(os.path.join(ROOT, "include"))
+            if f.endswith(".h")]
+    names = set()
+    for h in hdrs:
+        src = open(h).read()
+        src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+        for m in re.finditer(r"\b(bkmoo_[a-z0-9_]+)\s*\(", src):
+            names.add(m.group(1))
+    return sorted(names)
+
+
+def test_library_exports_every_declared_symbol():
+    names = _declared_symbols()
+    assert "bkmoo_resolve" in names and "bkmoo_plan" in names and "bkmoo_gram" in names
+    lib = ctypes.CDLL(bk.LIB_PATH)
+    for n in names:
+        assert hasattr(lib, n), n
+
+
+def test_version_and_status_strings():
+    assert bk.bkmoo_version() == 100
+    for code in range(8):
+        assert bk.bkmoo_status_string(code) != "unknown status"
+    assert bk.bkmoo_status_string(99) == "unknown status"
+
+
+def test_default_params():
+    p = bk.bkmoo_default_params()
+    assert p.max_iter == 256 and p.tol == 1e-12 and p.cagrad_c == 0.5
+    assert p.flags == bk.BKMOO_FLAG_CLOSED_FORM_K2 | bk.BKMOO_FLAG_POLISH
+
+
+def test_plan_bit_exact_vs_oracle_models():
+    for sizes, eb in [(inputs.gpt2_small_sizes(), 4), (inputs.llama32_1b_sizes(), 2),
+                      (inputs.qwen3_8b_sizes(), 2)]:
+        for bb in (inputs.MiB, 25 * inputs.MiB, 100 * inputs.MiB, 3 * 10**6 + 7):
+            np.testing.assert_array_equal(bk.bkmoo_plan(sizes, eb, bb), orc.plan(sizes, eb, bb))
+    for mib in inputs.SWEEP_BUCKET_MIB:
+        np.testing.assert_array_equal(bk.bkmoo_plan([10**9], 4, mib * inputs.MiB),
+                                      orc.plan([10**9], 4, mib * inputs.MiB))
+
+
+def test_plan_bit_exact_vs_oracle_random_and_golden():
+    import json
+    g = json.load(open(os.path.join(ROOT, "tests", "golden", "plan_cases.json")))
+    for c in g["cases"]:
+        assert bk.bkmoo_plan(c["sizes"], c["elem_bytes"], c["bucket_bytes"]).tolist() == c["offsets"]
+    rng = np.random.default_rng(0)
+    for _ in range(2000):
+        sizes = rng.integers(0, 100, size=int(rng.integers(0, 15))).tolist()
+        eb = int(rng.integers(1, 5))
+        bb = int(rng.integers(1, 300))
+        if bb // eb < 1:
+            continue
+        np.testing.assert_array_equal(bk.bkmoo_plan(sizes, eb, bb), orc.plan(sizes, eb, bb))
+
+
+def test_plan_buffer_too_small_and_invalid():
+    lib = bk.load()
+    sizes = np.array([10, 10, 10], dtype=np.int64)
+    nb_ = ctypes.c_int64(0)
+    out = np.zeros(2, dtype=np.int64)
+    r = lib.bkmoo_plan(sizes.ctypes.data, 3, 1, 10, out.ctypes.data, 2, ctypes.byref(nb_))
+    assert r == bk.BKMOO_ERR_BUFFER_TOO_SMALL and nb_.value == 3
+    assert lib.bkmoo_plan(sizes.ctypes.data, 3, 4, 3, None, 0, ctypes.byref(nb_)) == bk.BKMOO_ERR_INVALID
+    assert lib.bkmoo_plan(sizes.ctypes.data, 3, 0, 3, None, 0, ctypes.byref(nb_)) == bk.BKMOO_ERR_INVALID
+    bad = np.array([3, -1], dtype=np.int64)
+    assert lib.bkmoo_plan(bad.ctypes.data, 2, 1, 3, None, 0, ctypes.byref(nb_)) == bk.BKMOO_ERR_INVALID
+    assert lib.bkmoo_plan(sizes.ctypes.data, 3, 1, 3, None, 0, None) == bk.BKMOO_ERR_INVALID
+
+
+def test_workspace_size_layout():
+    off = orc.plan(inputs.qwen3_8b_sizes(), 2, 25 * inputs.MiB)
+    n4 = bk.bkmoo_workspace_size(4, bk.BKMOO_BF16, off)
+    n8 = bk.bkmoo_workspace_size(8, bk.BKMOO_BF16, off)
+    assert n8 > n4 > 0 and n4 % 256 == 0
+    # partials dominate: one fp64 triangle per 32768-element bf16 chunk
+    chunks = sum((int(off[b + 1] - off[b]) + 32767) // 32768 for b in range(len(off) - 1))
+    assert n4 >= chunks * 10 * 8
+    with pytest.raises(bk.BkmooError):
+        bk.bkmoo_workspace_size(0, bk.BKMOO_F32, off)
+    with pytest.raises(bk.BkmooError):
+        bk.bkmoo_workspace_size(17, bk.BKMOO_F32, off)
+    with pytest.raises(bk.BkmooError):
+        bk.bkmoo_workspace_size(4, 7, off)
+    with pytest.raises(bk.BkmooError):
+        bk.bkmoo_workspace_size(4, bk.BKMOO_F32, [0, 5, 5, 9])   # empty bucket
+    with pytest.raises(bk.BkmooError):
+        bk.bkmoo_workspace_size(4, bk.BKMOO_F32, [1, 5])          # must start at 0
+
+
+def test_resolve_rejects_bad_arguments_without_launch():
+    """Every check below fails before any CUDA call (fake, aligned addresses)."""
+    lib = bk.load()
+    off = np.array([0, 1000, 2500], dtype=np.int64)
+    base = 1 << 40
+    grads = (ctypes.c_void_p * 4)(*[base + i * (1 << 20) for i in range(4)])
+    ws = ctypes.c_void_p(base + (1 << 30))
+    out = ctypes.c_void_p(base + (1 << 31))
+    p = bk.bkmoo_default_params()
+
+    def call(**kw):
+        a = dict(grads=grads, K=4, dt=0, off=off.ctypes.data, B=2, rule=0, p=ctypes.byref(p),
+                 out=out, odt=0, w=None, st=None, ws=ws, wsb=1 << 30)
+        a.update(kw)
+        return lib.bkmoo_resolve(a["grads"], a["K"], a["dt"], a["off"], a["B"], a["rule"], a["p"],
+                                 a["out"], a["odt"], a["w"], a["st"], a["ws"], a["wsb"], None)
+
+    assert call(K=0) == bk.BKMOO_ERR_INVALID
+    assert call(K=17) == bk.BKMOO_ERR_INVALID
+    assert call(dt=2) == bk.BKMOO_ERR_INVALID
+    assert call(odt=5) == bk.BKMOO_ERR_INVALID
+    assert call(rule=4) == bk.BKMOO_ERR_INVALID
+    assert call(out=None) == bk.BKMOO_ERR_INVALID
+    assert call(out=ctypes.c_void_p(base + (1 << 31) + 4)) == bk.BKMOO_ERR_INVALID   # unaligned
+    assert call(ws=ctypes.c_void_p(base + (1 << 30) + 16)) == bk.BKMOO_ERR_INVALID  # ws not 256-B
+    assert call(wsb=64) == bk.BKMOO_ERR_WORKSPACE
+    bad = np.array([0, 1000, 900], dtype=np.int64)
+    assert call(off=bad.ctypes.data) == bk.BKMOO_ERR_INVALID
+    g2 = (ctypes.c_void_p * 4)(base, base + 8, base + (2 << 20), base + (3 << 20))
+    assert call(grads=g2) == bk.BKMOO_ERR_INVALID                                  # unaligned grad
+    # out overlapping a gradient without being exactly it
+    assert call(out=ctypes.c_void_p(base + 256)) == bk.BKMOO_ERR_INVALID
+    # in place over a gradient with another dtype
+    assert call(out=ctypes.c_void_p(base), odt=1) == bk.BKMOO_ERR_INVALID
+    q = bk.bkmoo_default_params()
+    q.cagrad_c = 1.0
+    assert call(p=ctypes.byref(q)) == bk.BKMOO_ERR_INVALID
+    q = bk.bkmoo_default_params()
+    q.max_iter = -1
+    assert call(p=ctypes.byref(q)) == bk.BKMOO_ERR_INVALID

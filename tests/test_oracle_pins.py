@@ -599,3 +599,25 @@ def test_synthetic_cosines_of_tiny_workload():
     for b, cos in enumerate(inputs.TINY_COSINES):
         G = orc.gram(vs, int(off[b]), int(off[b + 1] - off[b]))
         assert abs(G[0, 1] / math.sqrt(G[0, 0] * G[1, 1]) - cos) < 0.01
+
+
+def test_mgda_frank_wolfe_step_is_exact_line_search():
+    """One Frank-Wolfe step moves from the pair start towards the vertex of
+    least gradient to the minimiser along that segment (brute-force search)."""
+    rng = np.random.default_rng(37)
+    gam = np.linspace(0.0, 1.0, 100001)
+    for trial in range(30):
+        K = 3 + trial % 4
+        G = _gram_np(_rand_vectors(rng, K, 2 * K, corr=rng.uniform(-0.5, 0.9)))
+        a0, _ = orc.mgda_fw(G, 0, 0.0)
+        a1, done = orc.mgda_fw(G, 1, -1.0)
+        if done == 0:
+            continue
+        t = int(np.argmin(G @ a0))
+        e = np.zeros(K)
+        e[t] = 1.0
+        path = (1 - gam)[:, None] * a0[None, :] + gam[:, None] * e[None, :]
+        vals = np.einsum("ni,ij,nj->n", path, G, path)
+        j = int(np.argmin(vals))
+        assert _obj(G, a1) <= vals[j] + 1e-12 * G.max()
+        assert np.abs(a1 - path[j]).max() <= 2e-5
