@@ -9,7 +9,11 @@ Tolerances (per bucket):
      multiply-adds, each within 2^-24 of the running sum's magnitude, plus
      the fp32 rounding of beta); it only matters where d_oracle is near 0
      (opposed or linearly dependent gradients, Theorem 3.1 (a)), where a
-     pure relative error is undefined.
+     pure relative error is undefined.  bf16 output: round-to-nearest-even
+     has a relative error of at most 2^-8 per element, so
+     ||bf16(d) - d|| <= 2^-8 ||d|| always; 2e-3 is the rms that a long
+     bucket reaches (about 1.6e-3), so buckets under 4096 elements are held
+     to the hard bound 2^-8 instead.
   Gram: |G_gpu - G_oracle| <= 1e-5 sqrt(G_ii G_jj).  Each entry is summed in
      fp32 over at most 128 products per thread, then through a 5-level fp32
      shuffle tree, then in fp64; the fp32 stages contribute at most
@@ -34,7 +38,10 @@ def d_check(d_gpu, d_or, beta_or, g_norms, out_dt):
     nd = float(np.linalg.norm(d_or))
     err = float(np.linalg.norm(d_gpu - d_or))
     floor = (len(g_norms) + 2) * 2.0 ** -24 * float(np.dot(np.abs(beta_or), g_norms))
-    ok = err <= D_RTOL[out_dt] * nd + floor
+    rtol = D_RTOL[out_dt]
+    if out_dt == "bf16" and len(d_or) < 4096:
+        rtol = 2.0 ** -8
+    ok = err <= rtol * nd + floor
     return ok, (err / nd if nd > 0 else err)
 
 

@@ -82,7 +82,7 @@ def _check_against_oracle(w, rule, off, hv, out, beta, status, out_dt, seed=0, s
             assert np.abs(beta[b] - ref["beta"][b]).max() <= BETA_ATOL, (b, beta[b], ref["beta"][b])
         ok, e = d_check(d[lo:hi], ref["d"][lo:hi], ref["beta"][b], gn, out_dt)
         worst = max(worst, e)
-        assert ok, (rule, b, e)
+        assert ok, (rule, out_dt, b, e)
     return worst
 
 
