@@ -155,6 +155,38 @@ int bkmoo_gram(const void* const* grads, int32_t K, int32_t in_dtype,
                void* ws, size_t ws_bytes, void* stream);
 
 /*
+ * bkmoo_gram_noalloc -- bkmoo_gram without a workspace argument; it allocates
+ * no memory at all.  The paper has no counterpart: this is a service for
+ * callers that hold their input and output buffers but cannot get more
+ * device memory, for instance a hook inside a training framework whose
+ * device memory all belongs to the framework's caching allocator, or a C
+ * caller in a process where another component owns device allocation.
+ *
+ * Same arguments, results and determinism as bkmoo_gram (the same kernels
+ * run).  The scratch (bucket table and per-chunk partial sums) lives in a
+ * static device array of BKMOO_NOALLOC_SCRATCH_BYTES that every GPU which
+ * loads this library keeps until the process exits; the bucket table reaches
+ * it through kernel parameters, so no copy or allocating call is made.
+ * Limits: at most BKMOO_NOALLOC_MAX_BUCKETS buckets and a problem whose
+ * workspace (bkmoo_workspace_size) fits the array -- about 13 billion
+ * elements per language for K = 4 and 1 billion for K = 16 with bf16
+ * gradients (half as many with fp32); larger problems return
+ * BKMOO_ERR_WORKSPACE.
+ *
+ * The first call on each device (with that device current) looks up the
+ * array's device address once (cudaGetSymbolAddress); make that first call
+ * before any stream capture.  Every call shares the one array and rewrites
+ * the parts it reads, so results never depend on an earlier call; but calls
+ * whose work overlaps on the GPU (other streams or host threads on the same
+ * device) race on it and must be serialised by the caller.
+ */
+#define BKMOO_NOALLOC_SCRATCH_BYTES (32u << 20)
+#define BKMOO_NOALLOC_MAX_BUCKETS 4096
+int bkmoo_gram_noalloc(const void* const* grads, int32_t K, int32_t in_dtype,
+                       const int64_t* offsets, int64_t n_buckets, double* out_gram,
+                       void* stream);
+
+/*
  * bkmoo_resolve -- the resolve of Algorithm 1 for every bucket: Gram ->
  * rule -> d_b = sum_k beta_k g_k, written into the flat direction out_dir
  * (the concatenation of Section 3.2).

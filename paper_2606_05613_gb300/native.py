@@ -31,6 +31,8 @@ BKMOO_F32, BKMOO_BF16 = 0, 1
 BKMOO_FLAG_CLOSED_FORM_K2 = 0x1
 BKMOO_FLAG_POLISH = 0x2
 BKMOO_FLAG_FUSED = 0x4
+BKMOO_NOALLOC_SCRATCH_BYTES = 32 << 20
+BKMOO_NOALLOC_MAX_BUCKETS = 4096
 
 RULES = {"mgda": BKMOO_MGDA, "pcgrad": BKMOO_PCGRAD, "cagrad": BKMOO_CAGRAD, "mean": BKMOO_MEAN}
 
@@ -77,6 +79,8 @@ def load():
         lib.bkmoo_workspace_init.argtypes = [i32, i32, vp, i64, vp, sz, vp]
         lib.bkmoo_gram.restype = ctypes.c_int
         lib.bkmoo_gram.argtypes = [vp, i32, i32, vp, i64, vp, vp, sz, vp]
+        lib.bkmoo_gram_noalloc.restype = ctypes.c_int
+        lib.bkmoo_gram_noalloc.argtypes = [vp, i32, i32, vp, i64, vp, vp]
         lib.bkmoo_resolve.restype = ctypes.c_int
         lib.bkmoo_resolve.argtypes = [vp, i32, i32, vp, i64, i32, ctypes.POINTER(bkmoo_params),
                                       vp, i32, vp, vp, vp, sz, vp]
@@ -165,6 +169,18 @@ def bkmoo_gram(grads, offsets, out_gram, ws, stream=None):
                              len(off) - 1, out_gram.data_ptr(), ws.data_ptr(),
                              ws.numel() * ws.element_size(),
                              _stream_handle(stream, grads[0].device)), "bkmoo_gram")
+
+
+def bkmoo_gram_noalloc(grads, offsets, out_gram, stream=None):
+    """bkmoo_gram for callers that cannot allocate device memory: no
+    workspace; the scratch is a static device array of the library (see
+    include/bkmoo.h for its limits and the rule that overlapping calls race)."""
+    off = _offsets_array(offsets)
+    ptrs = _grad_ptrs(grads)
+    _check(load().bkmoo_gram_noalloc(ptrs, len(grads), _dtype_code(grads[0]), off.ctypes.data,
+                                     len(off) - 1, out_gram.data_ptr(),
+                                     _stream_handle(stream, grads[0].device)),
+           "bkmoo_gram_noalloc")
 
 
 def bkmoo_resolve(grads, offsets, rule, out_dir, ws, params=None, out_weights=None,
