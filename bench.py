@@ -44,6 +44,9 @@ def _args():
     ap.add_argument("--workload", default="qwen3-8b",
                     help="qwen3-8b | llama3.2-1b | gpt2-small | tiny | sweep-K-MiB")
     ap.add_argument("--rule", default="mgda", choices=["mgda", "pcgrad", "cagrad", "mean"])
+    ap.add_argument("--path", default="3pass", choices=["fused", "3pass"],
+                    help="fused: one persistent launch per step (re-read from L2); "
+                         "3pass: Gram, solve and combination launches")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=3)
@@ -299,6 +302,9 @@ def main():
     params = bk.bkmoo_default_params()
     if w.max_iter != 256:
         params.max_iter = w.max_iter
+    fused = a.path == "fused"
+    if fused:
+        params.flags |= bk.BKMOO_FLAG_FUSED
 
     def step(evs=None):
         if evs is not None:
@@ -350,10 +356,14 @@ def main():
     peak, peak_kind = _peaks()
     e_in = w.elem_bytes
     e_out = out.element_size()
-    kern = {"gram": (per[:, 0].mean(), w.K * e_in * N, "gram"),
-            "solve": (per[:, 1].mean(), None, "solve"),
-            "combine": (per[:, 2].mean(), (w.K * e_in + e_out) * N, "combine")}
-    dom = max(("gram", "combine"), key=lambda k: kern[k][0])
+    if fused:   # one launch: Gram + solve + combination, re-read from L2
+        kern = {"fused": (per[:, 0].mean(), (w.K * e_in + e_out) * N, "fused")}
+        dom = "fused"
+    else:
+        kern = {"gram": (per[:, 0].mean(), w.K * e_in * N, "gram"),
+                "solve": (per[:, 1].mean(), None, "solve"),
+                "combine": (per[:, 2].mean(), (w.K * e_in + e_out) * N, "combine")}
+        dom = max(("gram", "combine"), key=lambda k: kern[k][0])
     dms, dbytes, _ = kern[dom]
     achieved = dbytes / (dms * 1e-3) / GB
     tpe = _traffic_per_elem("%s_%s_k%d" % (dom, w.dtype, w.K))
@@ -376,13 +386,15 @@ def main():
                    "rule": a.rule, "n_elems_per_language": N, "n_buckets": B,
                    "bucket_bytes": w.bucket_bytes, "l2": "inputs (%.1f GB) >> L2, no flush"
                    % (grad_bytes / GB), "parallelism": "replicas" if world > 1 else "1 GPU",
-                   "path": "gram -> solve -> combine (3 launches)"},
+                   "path": ("fused: one persistent launch per step, combination re-reads "
+                            "each bucket from L2" if fused else
+                            "gram -> solve -> combine (3 launches)")},
         "roofline": roofline,
         "step_roofline": {"bytes_2k1": step_bytes_2k1, "bytes_k1": step_bytes_k1,
                           "frac_2k1_of_measured": step_bytes_2k1 / (ms_step * 1e-3) / GB / peak,
                           "frac_k1_of_measured": step_bytes_k1 / (ms_step * 1e-3) / GB / peak,
                           "frac_2k1_of_8tbs": step_bytes_2k1 / (ms_step * 1e-3) / GB / 8000.0},
-        "gpu_launches": 3 * a.steps,
+        "gpu_launches": (1 if fused else 3) * a.steps,
         "clocks": clk,
         "bucket_status_counts": {str(k): int((st == k).sum()) for k in sorted(set(st.tolist()))},
         "host_wall_ms_per_step": 1e3 * wall / a.steps,

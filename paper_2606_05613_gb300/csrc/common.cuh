@@ -17,6 +17,7 @@ constexpr int kWarps = kThreads / 32;
 constexpr int kVecPerThread = 16;          // 16-byte vectors per thread per Gram chunk
 constexpr uint32_t kMagic = 0x4f4d4b42u;   // "BKMO"
 constexpr int kSolveWarpsPerBlock = 4;
+constexpr int kFusedMaxCtas = 2048;        // upper bound of the fused grid
 
 __host__ __device__ constexpr int tri(int K) { return K * (K + 1) / 2; }
 __host__ __device__ constexpr int elems_per_vec(int dtype) { return dtype == BKMOO_F32 ? 4 : 8; }
@@ -45,7 +46,12 @@ struct WsLayout {
   size_t chunk_prefix;   // int64 [B + 1]   first Gram chunk of each bucket
   size_t partials;       // double [n_chunks][P] per-chunk Gram partials
   size_t beta;           // float [B][K]    coefficients of the last resolve
-  size_t total;
+  size_t total;          // end of the regions above
+  // fused path only (bkmoo_resolve with BKMOO_FLAG_FUSED):
+  size_t arrive;         // int32 [B]  streaming CTAs done with bucket b's Gram
+  size_t ready;          // int32 [B]  1 once beta of bucket b is written
+  size_t ring;           // double [2][kFusedMaxCtas][P] per-CTA partials
+  size_t total_fused;
 };
 
 __host__ __device__ inline size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
@@ -62,6 +68,13 @@ __host__ __device__ inline WsLayout ws_layout(int K, int64_t B, int64_t n_chunks
   L.beta = at;
   at = align256(at + sizeof(float) * (size_t)B * (size_t)K);
   L.total = at;
+  L.arrive = at;
+  at = align256(at + sizeof(int32_t) * (size_t)B);
+  L.ready = at;
+  at = align256(at + sizeof(int32_t) * (size_t)B);
+  L.ring = at;
+  at = align256(at + sizeof(double) * 2 * (size_t)kFusedMaxCtas * (size_t)tri(K));
+  L.total_fused = at;
   return L;
 }
 
@@ -82,6 +95,17 @@ struct PlanView {
   uint64_t plan_hash;
   int32_t K;
   int32_t in_dtype;
+};
+
+// The fused path's view: the plan plus the synchronisation arrays.
+struct FusedView {
+  PlanView v;
+  int32_t* arrive;
+  int32_t* ready;
+  double* ring;
+  float* out_weights;
+  int32_t* out_status;
+  int32_t n_stream;      // streaming CTAs; CTA n_stream is the solver
 };
 
 struct SolveParams {
@@ -180,6 +204,12 @@ const void* gram_partials_fn_bf16(int K);
 // Combine kernels, signature (GradPtrs, PlanView, void* out); combine_*.cu.
 const void* combine_fn_f32(int K, int dtype_out);
 const void* combine_fn_bf16(int K, int dtype_out);
+
+// Fused kernels, signature (GradPtrs, FusedView, SolveParams, void* out); fused_*.cu.
+const void* fused_fn_f32_k1_8(int K, int dtype_out);
+const void* fused_fn_f32_k9_16(int K, int dtype_out);
+const void* fused_fn_bf16_k1_8(int K, int dtype_out);
+const void* fused_fn_bf16_k9_16(int K, int dtype_out);
 
 // solve.cu
 cudaError_t launch_solve(const PlanView& v, const SolveParams& p, float* out_weights,

@@ -90,6 +90,41 @@ const void* gram_fn(int K, int dt) {
 const void* combine_fn(int K, int dti, int dto) {
   return dti == BKMOO_F32 ? combine_fn_f32(K, dto) : combine_fn_bf16(K, dto);
 }
+const void* fused_fn(int K, int dti, int dto) {
+  if (dti == BKMOO_F32) return K <= 8 ? fused_fn_f32_k1_8(K, dto) : fused_fn_f32_k9_16(K, dto);
+  return K <= 8 ? fused_fn_bf16_k1_8(K, dto) : fused_fn_bf16_k9_16(K, dto);
+}
+
+// The fused path: one cooperative (co-resident) launch; the last CTA solves.
+int launch_fused(const GradPtrs& g, const PlanView& v, const SolveParams& sp, void* ws,
+                 float* out_weights, int32_t* out_status, void* out, int dto, cudaStream_t s) {
+  const WsLayout L = ws_layout(v.K, v.n_buckets, v.n_chunks);
+  char* base = static_cast<char*>(ws);
+  if (cudaMemsetAsync(&v.hdr->status, 0, sizeof(int32_t), s) != cudaSuccess) return BKMOO_ERR_CUDA;
+  if (v.n_buckets == 0) return BKMOO_OK;
+  if (cudaMemsetAsync(base + L.arrive, 0, L.ring - L.arrive, s) != cudaSuccess)
+    return BKMOO_ERR_CUDA;
+  const void* fn = fused_fn(v.K, v.in_dtype, dto);
+  int grid = 0;
+  if (persistent_grid(fn, kThreads, &grid) != cudaSuccess) return BKMOO_ERR_CUDA;
+  if (grid > kFusedMaxCtas + 1) grid = kFusedMaxCtas + 1;
+  if (grid < 2) return BKMOO_ERR_CUDA;
+  FusedView f;
+  f.v = v;
+  f.arrive = reinterpret_cast<int32_t*>(base + L.arrive);
+  f.ready = reinterpret_cast<int32_t*>(base + L.ready);
+  f.ring = reinterpret_cast<double*>(base + L.ring);
+  f.out_weights = out_weights;
+  f.out_status = out_status;
+  f.n_stream = grid - 1;
+  GradPtrs ga = g;
+  SolveParams spa = sp;
+  void* outp = out;
+  void* args[] = {&ga, &f, &spa, &outp};
+  if (cudaLaunchCooperativeKernel(fn, dim3(grid), dim3(kThreads), args, 0, s) != cudaSuccess)
+    return BKMOO_ERR_CUDA;
+  return BKMOO_OK;
+}
 
 // Common checks of bkmoo_gram / bkmoo_resolve; fills the plan view.
 int prepare(const void* const* grads, int32_t K, int32_t dt, const int64_t* offsets,
@@ -102,7 +137,7 @@ int prepare(const void* const* grads, int32_t K, int32_t dt, const int64_t* offs
   const int64_t ch = chunk_elems(dt);
   const int64_t nch = count_chunks(offsets, B, ch);
   const WsLayout L = ws_layout(K, B, nch);
-  if (ws_bytes < L.total) return BKMOO_ERR_WORKSPACE;
+  if (ws_bytes < L.total_fused) return BKMOO_ERR_WORKSPACE;
   char* base = static_cast<char*>(ws);
   v->hdr = reinterpret_cast<WsHeader*>(base);
   v->offsets = reinterpret_cast<const int64_t*>(base + L.offsets);
@@ -195,7 +230,7 @@ int bkmoo_workspace_size(int32_t K, int32_t in_dtype, const int64_t* offsets,
   if (!bytes || K < 1 || K > kMaxK || !dtype_ok(in_dtype) || !offsets_ok(offsets, n_buckets))
     return BKMOO_ERR_INVALID;
   const int64_t nch = count_chunks(offsets, n_buckets, chunk_elems(in_dtype));
-  *bytes = ws_layout(K, n_buckets, nch).total;
+  *bytes = ws_layout(K, n_buckets, nch).total_fused;
   return BKMOO_OK;
 }
 
@@ -207,7 +242,7 @@ int bkmoo_workspace_init(int32_t K, int32_t in_dtype, const int64_t* offsets,
   const int64_t ch = chunk_elems(in_dtype);
   const int64_t nch = count_chunks(offsets, n_buckets, ch);
   const WsLayout L = ws_layout(K, n_buckets, nch);
-  if (ws_bytes < L.total) return BKMOO_ERR_WORKSPACE;
+  if (ws_bytes < L.total_fused) return BKMOO_ERR_WORKSPACE;
   // Host image of header + bucket table, copied in one transfer.
   std::vector<unsigned char> img(L.partials, 0);
   WsHeader h;
@@ -271,10 +306,6 @@ int bkmoo_resolve(const void* const* grads, int32_t K, int32_t in_dtype, const i
   }
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   cudaEvent_t* ev = static_cast<cudaEvent_t*>(prm.events);
-  if (ev && cudaEventRecord(ev[0], s) != cudaSuccess) return BKMOO_ERR_CUDA;
-  r = launch_gram_pass(g, v, s);
-  if (r != BKMOO_OK) return r;
-  if (ev && cudaEventRecord(ev[1], s) != cudaSuccess) return BKMOO_ERR_CUDA;
   SolveParams sp;
   sp.rule = rule;
   sp.max_iter = prm.max_iter;
@@ -283,6 +314,17 @@ int bkmoo_resolve(const void* const* grads, int32_t K, int32_t in_dtype, const i
   sp.seed = prm.seed;
   sp.step = prm.step;
   sp.flags = prm.flags;
+  if (ev && cudaEventRecord(ev[0], s) != cudaSuccess) return BKMOO_ERR_CUDA;
+  if (prm.flags & BKMOO_FLAG_FUSED) {
+    r = launch_fused(g, v, sp, ws, out_weights, out_status, out_dir, out_dtype, s);
+    if (r != BKMOO_OK) return r;
+    for (int i = 1; i < 4; ++i)
+      if (ev && cudaEventRecord(ev[i], s) != cudaSuccess) return BKMOO_ERR_CUDA;
+    return BKMOO_OK;
+  }
+  r = launch_gram_pass(g, v, s);
+  if (r != BKMOO_OK) return r;
+  if (ev && cudaEventRecord(ev[1], s) != cudaSuccess) return BKMOO_ERR_CUDA;
   if (launch_solve(v, sp, out_weights, out_status, s) != cudaSuccess) return BKMOO_ERR_CUDA;
   if (ev && cudaEventRecord(ev[2], s) != cudaSuccess) return BKMOO_ERR_CUDA;
   if (v.n_chunks == 0) {

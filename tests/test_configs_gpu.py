@@ -161,12 +161,16 @@ def test_qwen3_8b_k4_bf16_mgda_cagrad():
     samples = _spread(B, 3) + conflicted[:3]
     res = None
     out = None
-    for rule in ("mgda", "cagrad"):
-        res, out, beta, st = _resolve(w, off, grads, rule, res=res, out=out)
-        assert (st == 0).all(), np.unique(st, return_counts=True)
-        _check_sampled(w, off, grads, out, beta, st, rule, samples)
-        if rule == "mgda":
-            _mgda_properties(_gram_all(res, grads, w, off), beta)
+    for fused in (False, True):
+        for rule in ("mgda", "cagrad"):
+            p = bk.bkmoo_default_params()
+            if fused:
+                p.flags |= bk.BKMOO_FLAG_FUSED
+            res, out, beta, st = _resolve(w, off, grads, rule, p, res=res, out=out)
+            assert (st == 0).all(), np.unique(st, return_counts=True)
+            _check_sampled(w, off, grads, out, beta, st, rule, samples)
+            if rule == "mgda":
+                _mgda_properties(_gram_all(res, grads, w, off), beta)
 
 
 @pytest.mark.parametrize("K", inputs.SWEEP_K)

@@ -263,3 +263,77 @@ def test_all_zero_bucket_gives_zero_direction():
         res.resolve(grads, rule, out)
         torch.cuda.synchronize()
         assert torch.count_nonzero(out).item() == 0
+
+
+# ---------------------------------------------------------------------------
+# fused path (BKMOO_FLAG_FUSED): one persistent launch per resolve
+# ---------------------------------------------------------------------------
+
+def _fused_params(seed=0, step=0, flags=None):
+    p = bk.bkmoo_default_params()
+    p.seed, p.step = seed, step
+    p.flags = (p.flags if flags is None else flags) | bk.BKMOO_FLAG_FUSED
+    return p
+
+
+@pytest.mark.parametrize("rule", ["mgda", "pcgrad", "cagrad", "mean"])
+@pytest.mark.parametrize("dt,out_dt", [("f32", "f32"), ("bf16", "bf16"), ("bf16", "f32")])
+@pytest.mark.parametrize("K", [1, 2, 3, 4, 5, 8, 16])
+def test_fused_resolve_parity(rule, dt, out_dt, K):
+    w = _workload(K, dt, RAGGED, 150000, seed=60 + K, flip=0.2)
+    off, hv, out, beta, status, _ = _run(w, rule, out_dt, params=_fused_params(5, 9))
+    _check_against_oracle(w, rule, off, hv, out, beta, status, out_dt, seed=5, step=9)
+
+
+def test_fused_tiny_buckets_and_empty_slices():
+    """Buckets far smaller than the grid (most slices empty) and every
+    head / tail length."""
+    sizes = [1, 2, 3, 4, 5, 6, 7, 8, 9, 15, 16, 17, 31, 33, 1000, 8191, 8193, 300001]
+    for dt in ("f32", "bf16"):
+        w = _workload(3, dt, sizes, 400000)
+        off = np.concatenate([[0], np.cumsum(list(reversed(sizes)))]).astype(np.int64)
+        grads = inputs.generate(w, off, DEV)
+        hv = [inputs.host_view(g) for g in grads]
+        B = len(off) - 1
+        res = bk.Resolver(3, _tdt(dt), off, DEV)
+        for rule in ("mgda", "pcgrad", "cagrad"):
+            out = torch.empty(int(off[-1]), dtype=_tdt(dt), device=DEV)
+            beta = torch.empty(B, 3, device=DEV)
+            status = torch.empty(B, dtype=torch.int32, device=DEV)
+            res.resolve(grads, rule, out, params=_fused_params(), out_weights=beta,
+                        out_status=status)
+            torch.cuda.synchronize()
+            assert res.status() == 0
+            _check_against_oracle(w, rule, off, hv, out, beta.cpu().numpy(),
+                                  status.cpu().numpy(), dt)
+
+
+def test_fused_deterministic_and_matches_three_pass():
+    w = _workload(4, "bf16", RAGGED * 3, 250000, seed=8)
+    off, hv, out_f, beta_f, _, res = _run(w, "mgda", "f32", params=_fused_params())
+    o1 = out_f.clone()
+    grads = inputs.generate(w, off, DEV)
+    res.resolve(grads, "mgda", out_f, params=_fused_params())
+    torch.cuda.synchronize()
+    assert torch.equal(o1, out_f)                     # run to run
+    _, _, out_3, beta_3, _, _ = _run(w, "mgda", "f32")
+    np.testing.assert_allclose(beta_f, beta_3, atol=1e-5)
+    d3 = out_3.cpu().numpy().astype(np.float64)
+    df = o1.cpu().numpy().astype(np.float64)
+    assert np.linalg.norm(df - d3) <= 1e-5 * np.linalg.norm(d3)
+
+
+def test_fused_workspace_mismatch_is_detected():
+    w = _workload(2, "f32", [40000, 40000], 40000, seed=6)
+    off = bk.bkmoo_plan(w.param_sizes, w.elem_bytes, w.bucket_bytes)
+    grads = inputs.generate(w, off, DEV)
+    res = bk.Resolver(2, torch.float32, off, DEV)
+    other = np.array([0, 30000, 80000], dtype=np.int64)
+    out = torch.full_like(grads[0], 7.0)
+    status = torch.empty(2, dtype=torch.int32, device=DEV)
+    bk.bkmoo_resolve(grads, other, "mgda", out, res.ws, params=_fused_params(), out_status=status)
+    assert bk.bkmoo_workspace_status(res.ws) == bk.BKMOO_ERR_WORKSPACE
+    assert (status.cpu().numpy() == bk.BKMOO_ERR_WORKSPACE).all()
+    assert bool((out == 7.0).all())
+    res.resolve(grads, "mgda", out, params=_fused_params())
+    assert res.status() == 0
