@@ -106,6 +106,8 @@ struct FusedView {
   float* out_weights;
   int32_t* out_status;
   int32_t n_stream;      // streaming CTAs; CTA n_stream is the solver
+  int32_t lookahead;     // how far (in 1/1024 of a piece) the Gram of bucket
+                         // b+1 may lead the combination of bucket b
 };
 
 struct SolveParams {

@@ -75,6 +75,16 @@ __device__ __forceinline__ int ld_acquire(const int32_t* p) {
   asm volatile("ld.acquire.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
   return v;
 }
+// A poll that does not order later loads (so it can be issued before a
+// streaming step and read after it); pair a positive poll with fence_acquire.
+__device__ __forceinline__ int ld_relaxed(const int32_t* p) {
+  int v;
+  asm volatile("ld.relaxed.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(p));
+  return v;
+}
+__device__ __forceinline__ void fence_acquire() {
+  asm volatile("fence.acq_rel.gpu;" ::: "memory");
+}
 
 __device__ __forceinline__ uint64_t global_ns() {
   uint64_t t;
@@ -117,31 +127,47 @@ __device__ __forceinline__ void fused_slice(const PlanView& v, int64_t b, int i,
 template <int K>
 __device__ __noinline__ void fused_solver_cta(const FusedView& f, const SolveParams& prm) {
   constexpr int P = tri(K);
+  constexpr int STRIPES = kThreads / P > 0 ? kThreads / P : 1;
   __shared__ double G[K * K];
+  __shared__ float Gf[K * K];
   __shared__ double part[kThreads];
   __shared__ double beta_sh[K];
   __shared__ int go;
   const PlanView& v = f.v;
   const int n = f.n_stream;
-  // thread t sums stripe t / P of entry t % P over the CTAs of that stripe
-  constexpr int STRIPES = kThreads / P > 0 ? kThreads / P : 1;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   for (int64_t b = 0; b < v.n_buckets; ++b) {
     if (threadIdx.x == 0) go = fused_wait(f.arrive + b, n, v.hdr) ? 1 : 0;
     __syncthreads();
     if (!go) return;
+    // fixed-order reduction of the n CTA partials: thread t sums entry t % P
+    // over stripe t / P of the CTAs with four interleaved accumulators, then
+    // thread e adds its STRIPES stripe sums in order
     const double* ring = f.ring + (size_t)(b & 1) * kFusedMaxCtas * P;
     if ((int)threadIdx.x < STRIPES * P) {
       const int e = threadIdx.x % P, st = threadIdx.x / P;
       const int c0 = (int)((int64_t)n * st / STRIPES), c1 = (int)((int64_t)n * (st + 1) / STRIPES);
-      double t = 0.0;
-      for (int c = c0; c < c1; ++c) t += __ldcg(ring + (size_t)c * P + e);
-      part[threadIdx.x] = t;
+      double t0 = 0.0, t1 = 0.0, t2 = 0.0, t3 = 0.0;
+      int c = c0;
+      for (; c + 3 < c1; c += 4) {
+        t0 += __ldcg(ring + (size_t)c * P + e);
+        t1 += __ldcg(ring + (size_t)(c + 1) * P + e);
+        t2 += __ldcg(ring + (size_t)(c + 2) * P + e);
+        t3 += __ldcg(ring + (size_t)(c + 3) * P + e);
+      }
+      for (; c < c1; ++c) t0 += __ldcg(ring + (size_t)c * P + e);
+      part[threadIdx.x] = (t0 + t1) + (t2 + t3);
     }
     __syncthreads();
     if ((int)threadIdx.x < P) {
-      double t = 0.0;
-      for (int st = 0; st < STRIPES; ++st) t += part[st * P + threadIdx.x];
+      double t0 = 0.0, t1 = 0.0;
+      int st = 0;
+      for (; st + 1 < STRIPES; st += 2) {
+        t0 += part[st * P + threadIdx.x];
+        t1 += part[(st + 1) * P + threadIdx.x];
+      }
+      if (st < STRIPES) t0 += part[st * P + threadIdx.x];
+      const double t = t0 + t1;
       int i = 0, r = threadIdx.x;
       while (r >= K - i) {
         r -= K - i;
@@ -152,7 +178,7 @@ __device__ __noinline__ void fused_solver_cta(const FusedView& f, const SolvePar
     }
     __syncthreads();
     if (warp == 0) {
-      const int st = solver::solve_bucket_warp(K, G, prm, b, beta_sh, lane);
+      const int st = solver::solve_bucket_warp(K, G, Gf, prm, b, beta_sh, lane);
       if (lane < K) {
         const float fb = (float)beta_sh[lane];
         v.beta[b * K + lane] = fb;
@@ -171,23 +197,40 @@ __device__ __noinline__ void fused_solver_cta(const FusedView& f, const SolvePar
 }
 
 // Resident CTAs per SM the register budget is capped for: the streaming
-// loops need about 48 (K <= 4) and 128 (K <= 8) registers per thread; the
+// loops need up to 128 (K <= 4) and 255 (K > 4) registers per thread; the
 // solver code shares the kernel and spills instead of lowering occupancy.
 template <int K>
 struct FusedMinBlocks {
-  static constexpr int value = K <= 4 ? 4 : (K <= 8 ? 2 : 1);
+  static constexpr int value = K <= 4 ? 2 : 1;
 };
+
+// Piece of bucket b streamed by warp w of CTA cta: the CTA's slice cut in
+// kWarps equal, 16-byte-aligned pieces.
+template <int EPV>
+__device__ __forceinline__ void warp_piece(const PlanView& v, int64_t b, int cta, int n, int w,
+                                           int64_t* lo, int64_t* hi) {
+  int64_t a, z;
+  fused_slice<EPV>(v, b, cta, n, &a, &z);
+  int64_t ps = (z - a + kWarps - 1) / kWarps;
+  ps = (ps + EPV - 1) / EPV * EPV;
+  int64_t l = a + (int64_t)w * ps;
+  if (l > z) l = z;
+  int64_t h = l + ps;
+  if (h > z) h = z;
+  *lo = l;
+  *hi = h;
+}
 
 template <int K, int DT, int DTO>
 __global__ void __launch_bounds__(kThreads, FusedMinBlocks<K>::value)
     fused_resolve_kernel(const GradPtrs g, const FusedView f, const SolveParams prm, void* out) {
   constexpr int P = tri(K);
+  constexpr int NP = (P + 31) / 32;       // fp64 accumulators per lane
   constexpr int EPV = elems_per_vec(DT);
   constexpr int IB = 16 / EPV;
-  constexpr int STEP = 2;                 // vectors per thread per Gram / combine step
-  __shared__ float red[kWarps][P];
-  __shared__ float beta_sh[K];
-  __shared__ int s_go;
+  constexpr int STEP = K <= 2 ? 4 : 2;    // vectors per lane per Gram / combination step
+  __shared__ double part_sm[2][kWarps][P];
+  __shared__ int cnt_sm[2];
   const PlanView& v = f.v;
   if (!header_ok(v)) {
     if (blockIdx.x == 0 && threadIdx.x == 0) record_error(v.hdr, BKMOO_ERR_WORKSPACE);
@@ -200,173 +243,206 @@ __global__ void __launch_bounds__(kThreads, FusedMinBlocks<K>::value)
     fused_solver_cta<K>(f, prm);
     return;
   }
+  if (threadIdx.x < 2) cnt_sm[threadIdx.x] = 0;
+  __syncthreads();   // the only CTA-wide barrier; every warp runs on its own below
+
   const int cta = blockIdx.x, n = f.n_stream;
+  const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
   const int64_t B = v.n_buckets;
   const uint64_t keep = policy_evict_last(), last_use = policy_evict_first();
 
-  // Gram stepper over bucket gb (this CTA's slice)
-  int64_t gb = 0, g_lo = 0, g_vs = 0, g_nv = 0, g_next = 0;
+  int64_t gb = 0, g_vs = 0, g_nv = 0, g_next = 0;
   int g_pend = 0;
   bool g_open = false;
   float acc[P];
 #pragma unroll
   for (int p = 0; p < P; ++p) acc[p] = 0.0f;
-  double acc64 = 0.0;
-  // combination stepper over bucket cb
-  int64_t cb = 0, c_lo = 0, c_hi = 0, c_vs = 0, c_nv = 0, c_next = 0;
+  double acc64[NP];
+#pragma unroll
+  for (int i = 0; i < NP; ++i) acc64[i] = 0.0;
+
+  int64_t cb = 0, c_vs = 0, c_nv = 0, c_next = 0;
   bool c_open = false;
   float beta[K];
+#pragma unroll
+  for (int k = 0; k < K; ++k) beta[k] = 0.0f;
 
   while (cb < B) {
-    // one Gram step, at most one bucket ahead of the combination
-    const bool can_gram = gb < B && gb <= cb + 1;
-    if (can_gram) {
+    // poll for beta of bucket cb now; read the answer after the Gram step
+    const bool want = !c_open && cb < gb;
+    int flag = 0;
+    if (want && lane == 0) flag = ld_relaxed(f.ready + cb);
+
+    // ---- one Gram step of bucket gb: at most one bucket ahead of cb, and
+    // when ahead, at most `lookahead` of a piece ahead of the combination
+    // of cb, so that both buckets' unconsumed lines fit in L2
+    bool gram_ok = gb < B && gb <= cb + 1;
+    if (gram_ok && gb == cb + 1 && g_open) {
+      const int64_t lead = (g_nv * f.lookahead) >> 10;
+      const int64_t follow = c_open ? (c_next * g_nv) / (c_nv > 0 ? c_nv : 1) : 0;
+      gram_ok = g_next < follow + lead;
+    }
+    if (gram_ok) {
       if (!g_open) {
-        int64_t hi;
-        fused_slice<EPV>(v, gb, cta, n, &g_lo, &hi);
-        g_vs = (g_lo + EPV - 1) / EPV * EPV;
+        int64_t lo, hi;
+        warp_piece<EPV>(v, gb, cta, n, wid, &lo, &hi);
+        g_vs = (lo + EPV - 1) / EPV * EPV;
         if (g_vs > hi) g_vs = hi;
         int64_t ve = hi / EPV * EPV;
         if (ve < g_vs) ve = g_vs;
         g_nv = (ve - g_vs) / EPV;
-        const int nh = (int)(g_vs - g_lo), nt = (int)(hi - ve);
-        if ((int)threadIdx.x < nh + nt) {
-          const int64_t idx = (int)threadIdx.x < nh ? g_lo + threadIdx.x : ve + (threadIdx.x - nh);
+        const int nh = (int)(g_vs - lo), nt = (int)(hi - ve);
+        if (lane < nh + nt) {
+          const int64_t idx = lane < nh ? lo + lane : ve + (lane - nh);
           gram_accumulate_scalar<K, DT>(acc, g, idx);
         }
         g_next = 0;
         g_pend = 0;
-        acc64 = 0.0;
         g_open = true;
       }
-      {
-        uint4 r[STEP][K];
+      uint4 r[STEP][K];
 #pragma unroll
-        for (int j = 0; j < STEP; ++j) {
-          const int64_t idx = g_next + threadIdx.x + (int64_t)j * kThreads;
-          if (idx < g_nv) {
+      for (int j = 0; j < STEP; ++j) {
+        const int64_t idx = g_next + lane + 32 * j;
+        if (idx < g_nv) {
 #pragma unroll
-            for (int k = 0; k < K; ++k)
-              r[j][k] = ld16_policy_nc(static_cast<const char*>(g.p[k]) + (g_vs + idx * EPV) * IB, keep);
-          }
+          for (int k = 0; k < K; ++k)
+            r[j][k] = ld16_policy_nc(static_cast<const char*>(g.p[k]) + (g_vs + idx * EPV) * IB, keep);
         }
-#pragma unroll
-        for (int j = 0; j < STEP; ++j)
-          if (g_next + threadIdx.x + (int64_t)j * kThreads < g_nv) gram_accumulate<K, DT>(acc, r[j]);
       }
-      g_next += (int64_t)STEP * kThreads;
+#pragma unroll
+      for (int j = 0; j < STEP; ++j)
+        if (g_next + lane + 32 * j < g_nv) gram_accumulate<K, DT>(acc, r[j]);
+      g_next += 32 * STEP;
       g_pend += STEP;
       const bool done = g_next >= g_nv;
-      if (done || g_pend >= kVecPerThread) {   // fixed-order reduction of the sub-slice
-        const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+      if (done || g_pend >= kVecPerThread) {
+        // fixed butterfly over the warp; lane p % 32 keeps entry p in fp64
 #pragma unroll
         for (int p = 0; p < P; ++p) {
           float x = acc[p];
-          x += __shfl_down_sync(0xffffffffu, x, 16);
-          x += __shfl_down_sync(0xffffffffu, x, 8);
-          x += __shfl_down_sync(0xffffffffu, x, 4);
-          x += __shfl_down_sync(0xffffffffu, x, 2);
-          x += __shfl_down_sync(0xffffffffu, x, 1);
-          if (lane == 0) red[warp][p] = x;
+          x += __shfl_xor_sync(0xffffffffu, x, 16);
+          x += __shfl_xor_sync(0xffffffffu, x, 8);
+          x += __shfl_xor_sync(0xffffffffu, x, 4);
+          x += __shfl_xor_sync(0xffffffffu, x, 2);
+          x += __shfl_xor_sync(0xffffffffu, x, 1);
+          if ((p & 31) == lane) acc64[p >> 5] += (double)x;
           acc[p] = 0.0f;
         }
-        __syncthreads();
-        if ((int)threadIdx.x < P) {
-          double t = 0.0;
-#pragma unroll
-          for (int w = 0; w < kWarps; ++w) t += (double)red[w][threadIdx.x];
-          acc64 += t;
-        }
         g_pend = 0;
-        if (done) {
-          double* ring = f.ring + (size_t)(gb & 1) * kFusedMaxCtas * P + (size_t)cta * P;
-          if ((int)threadIdx.x < P) {
-            ring[threadIdx.x] = acc64;
+      }
+      if (done) {
+        // combine the CTA's 8 warp partials in a fixed order; the last warp
+        // to finish publishes the CTA's partial and arrives
+        const int slot = (int)(gb & 1);
+#pragma unroll
+        for (int i = 0; i < NP; ++i)
+          if (lane + 32 * i < P) part_sm[slot][wid][lane + 32 * i] = acc64[i];
+        __threadfence_block();
+        __syncwarp();
+        int last = 0;
+        if (lane == 0) last = (atomicAdd(&cnt_sm[slot], 1) == kWarps - 1) ? 1 : 0;
+        last = __shfl_sync(0xffffffffu, last, 0);
+        if (last) {
+          __threadfence_block();
+          double* ring = f.ring + (size_t)slot * kFusedMaxCtas * P + (size_t)cta * P;
+#pragma unroll
+          for (int i = 0; i < NP; ++i) {
+            const int p = lane + 32 * i;
+            if (p < P) {
+              double t = 0.0;
+#pragma unroll
+              for (int w = 0; w < kWarps; ++w) t += ((volatile double*)part_sm[slot][w])[p];
+              ring[p] = t;
+            }
+          }
+          __threadfence();
+          __syncwarp();
+          if (lane == 0) {
+            cnt_sm[slot] = 0;
             __threadfence();
+            atomicAdd(f.arrive + gb, 1);
           }
         }
-        __syncthreads();
-        if (done) {
-          if (threadIdx.x == 0) atomicAdd(f.arrive + gb, 1);
-          ++gb;
-          g_open = false;
-        }
+#pragma unroll
+        for (int i = 0; i < NP; ++i) acc64[i] = 0.0;
+        ++gb;
+        g_open = false;
       }
     }
 
-    // combination of bucket cb once its beta is ready
-    if (cb < gb) {
-      if (!c_open) {
-        if (threadIdx.x == 0) {
-          int go;
-          if (can_gram && gb <= cb + 1 && gb < B) {   // more Gram work to overlap: just look
-            go = ld_acquire(f.ready + cb) >= 1 ? 1 : 0;
-            if (!go && *(volatile int32_t*)&v.hdr->status != 0) go = -1;
-          } else {
-            go = fused_wait(f.ready + cb, 1, v.hdr) ? 1 : -1;
-          }
-          if (go == 1) {
+    // ---- open the combination of bucket cb once its beta is ready
+    if (want) {
+      flag = __shfl_sync(0xffffffffu, flag, 0);
+      bool more = gb < B && gb <= cb + 1;
+      if (more && gb == cb + 1 && g_open) more = g_next < ((g_nv * f.lookahead) >> 10);
+      if (!flag && !more) {   // nothing left to overlap: wait
+        int ok = 0;
+        if (lane == 0) ok = fused_wait(f.ready + cb, 1, v.hdr) ? 1 : 0;
+        if (!__shfl_sync(0xffffffffu, ok, 0)) return;
+        flag = 1;
+      }
+      if (flag) {
+        fence_acquire();
+        float bl = lane < K ? __ldcg(v.beta + cb * K + lane) : 0.0f;
 #pragma unroll
-            for (int k = 0; k < K; ++k) beta_sh[k] = __ldcg(v.beta + cb * K + k);
-          }
-          s_go = go;
+        for (int k = 0; k < K; ++k) beta[k] = __shfl_sync(0xffffffffu, bl, k);
+        int64_t lo, hi;
+        warp_piece<EPV>(v, cb, cta, n, wid, &lo, &hi);
+        c_vs = (lo + EPV - 1) / EPV * EPV;
+        if (c_vs > hi) c_vs = hi;
+        int64_t ve = hi / EPV * EPV;
+        if (ve < c_vs) ve = c_vs;
+        c_nv = (ve - c_vs) / EPV;
+        const int nh = (int)(c_vs - lo), nt = (int)(hi - ve);
+        if (lane < nh + nt) {
+          const int64_t idx = lane < nh ? lo + lane : ve + (lane - nh);
+          float t = 0.0f;
+#pragma unroll
+          for (int k = 0; k < K; ++k) t = fmaf(beta[k], load_scalar<DT>(g.p[k], idx), t);
+          store_scalar<DTO>(out, idx, t);
         }
-        __syncthreads();
-        const int go = s_go;
-        if (go < 0) return;
-        if (go == 1) {
+        c_next = 0;
+        c_open = true;
+      } else if (*(volatile int32_t*)&v.hdr->status != 0) {
+        return;
+      }
+    }
+
+    // ---- one combination step of bucket cb, from the end of the piece back
+    // to its start: the lines the Gram pass read last are read first, so
+    // an LRU L2 still holds them even when the bucket and its output
+    // together slightly exceed the cache
+    if (c_open) {
+      uint4 r[STEP][K];
 #pragma unroll
-          for (int k = 0; k < K; ++k) beta[k] = beta_sh[k];
-          fused_slice<EPV>(v, cb, cta, n, &c_lo, &c_hi);
-          c_vs = (c_lo + EPV - 1) / EPV * EPV;
-          if (c_vs > c_hi) c_vs = c_hi;
-          int64_t ve = c_hi / EPV * EPV;
-          if (ve < c_vs) ve = c_vs;
-          c_nv = (ve - c_vs) / EPV;
-          const int nh = (int)(c_vs - c_lo), nt = (int)(c_hi - ve);
-          if ((int)threadIdx.x < nh + nt) {
-            const int64_t idx = (int)threadIdx.x < nh ? c_lo + threadIdx.x : ve + (threadIdx.x - nh);
+      for (int j = 0; j < STEP; ++j) {
+        const int64_t idx = c_nv - 1 - (c_next + lane + 32 * j);
+        if (idx >= 0) {
+#pragma unroll
+          for (int k = 0; k < K; ++k)
+            r[j][k] = ld16_policy(static_cast<const char*>(g.p[k]) + (c_vs + idx * EPV) * IB, last_use);
+        }
+      }
+#pragma unroll
+      for (int j = 0; j < STEP; ++j) {
+        const int64_t idx = c_nv - 1 - (c_next + lane + 32 * j);
+        if (idx >= 0) {
+          float y[EPV];
+#pragma unroll
+          for (int q = 0; q < EPV; ++q) {
             float t = 0.0f;
 #pragma unroll
-            for (int k = 0; k < K; ++k) t = fmaf(beta[k], load_scalar<DT>(g.p[k], idx), t);
-            store_scalar<DTO>(out, idx, t);
+            for (int k = 0; k < K; ++k) t = fmaf(beta[k], vec_elem<DT>(r[j][k], q), t);
+            y[q] = t;
           }
-          c_next = 0;
-          c_open = true;
+          store_out<DTO>(out, c_vs + idx * EPV, y, EPV);
         }
-        __syncthreads();
       }
-      if (c_open) {
-        uint4 r[STEP][K];
-#pragma unroll
-        for (int j = 0; j < STEP; ++j) {
-          const int64_t idx = c_next + threadIdx.x + (int64_t)j * kThreads;
-          if (idx < c_nv) {
-#pragma unroll
-            for (int k = 0; k < K; ++k)
-              r[j][k] = ld16_policy(static_cast<const char*>(g.p[k]) + (c_vs + idx * EPV) * IB, last_use);
-          }
-        }
-#pragma unroll
-        for (int j = 0; j < STEP; ++j) {
-          const int64_t idx = c_next + threadIdx.x + (int64_t)j * kThreads;
-          if (idx < c_nv) {
-            float y[EPV];
-#pragma unroll
-            for (int q = 0; q < EPV; ++q) {
-              float t = 0.0f;
-#pragma unroll
-              for (int k = 0; k < K; ++k) t = fmaf(beta[k], vec_elem<DT>(r[j][k], q), t);
-              y[q] = t;
-            }
-            store_out<DTO>(out, c_vs + idx * EPV, y, EPV);
-          }
-        }
-        c_next += (int64_t)STEP * kThreads;
-        if (c_next >= c_nv) {
-          c_open = false;
-          ++cb;
-        }
+      c_next += 32 * STEP;
+      if (c_next >= c_nv) {
+        c_open = false;
+        ++cb;
       }
     }
   }

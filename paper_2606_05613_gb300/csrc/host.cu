@@ -97,7 +97,8 @@ const void* fused_fn(int K, int dti, int dto) {
 
 // The fused path: one cooperative (co-resident) launch; the last CTA solves.
 int launch_fused(const GradPtrs& g, const PlanView& v, const SolveParams& sp, void* ws,
-                 float* out_weights, int32_t* out_status, void* out, int dto, cudaStream_t s) {
+                 float* out_weights, int32_t* out_status, void* out, int dto,
+                 double bucket_bytes_max, cudaStream_t s) {
   const WsLayout L = ws_layout(v.K, v.n_buckets, v.n_chunks);
   char* base = static_cast<char*>(ws);
   if (cudaMemsetAsync(&v.hdr->status, 0, sizeof(int32_t), s) != cudaSuccess) return BKMOO_ERR_CUDA;
@@ -111,12 +112,26 @@ int launch_fused(const GradPtrs& g, const PlanView& v, const SolveParams& sp, vo
   if (grid < 2) return BKMOO_ERR_CUDA;
   FusedView f;
   f.v = v;
+  f.lookahead = 0;
   f.arrive = reinterpret_cast<int32_t*>(base + L.arrive);
   f.ready = reinterpret_cast<int32_t*>(base + L.ready);
   f.ring = reinterpret_cast<double*>(base + L.ring);
   f.out_weights = out_weights;
   f.out_status = out_status;
   f.n_stream = grid - 1;
+  // Look-ahead that keeps one bucket plus the part of the next one already
+  // read within 90 % of L2 (at least 1/20 of a bucket, at most a whole one).
+  {
+    int dev = 0, l2 = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&l2, cudaDevAttrL2CacheSize, dev) != cudaSuccess)
+      return BKMOO_ERR_CUDA;
+    const double wmax = bucket_bytes_max;
+    double la = (0.9 * (double)l2 - wmax) / (wmax > 0 ? wmax : 1.0);
+    if (la < 0.05) la = 0.05;
+    if (la > 1.0) la = 1.0;
+    f.lookahead = (int32_t)(la * 1024.0);
+  }
   GradPtrs ga = g;
   SolveParams spa = sp;
   void* outp = out;
@@ -316,7 +331,11 @@ int bkmoo_resolve(const void* const* grads, int32_t K, int32_t in_dtype, const i
   sp.flags = prm.flags;
   if (ev && cudaEventRecord(ev[0], s) != cudaSuccess) return BKMOO_ERR_CUDA;
   if (prm.flags & BKMOO_FLAG_FUSED) {
-    r = launch_fused(g, v, sp, ws, out_weights, out_status, out_dir, out_dtype, s);
+    int64_t nmax = 0;
+    for (int64_t b = 0; b < n_buckets; ++b)
+      if (offsets[b + 1] - offsets[b] > nmax) nmax = offsets[b + 1] - offsets[b];
+    r = launch_fused(g, v, sp, ws, out_weights, out_status, out_dir, out_dtype,
+                     (double)nmax * K * elem_bytes(in_dtype), s);
     if (r != BKMOO_OK) return r;
     for (int i = 1; i < 4; ++i)
       if (ev && cudaEventRecord(ev[i], s) != cudaSuccess) return BKMOO_ERR_CUDA;

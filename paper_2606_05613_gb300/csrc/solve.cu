@@ -14,6 +14,7 @@ __global__ void __launch_bounds__(32 * kSolveWarpsPerBlock)
                  int32_t* out_status) {
   __shared__ double Gs[kSolveWarpsPerBlock][kMaxK * kMaxK];
   __shared__ double Bs[kSolveWarpsPerBlock][kMaxK];
+  __shared__ float Fs[kSolveWarpsPerBlock][kMaxK * kMaxK];
   const int lane = threadIdx.x & 31, wi = threadIdx.x >> 5;
   const int64_t b = (int64_t)blockIdx.x * kSolveWarpsPerBlock + wi;
   if (b >= v.n_buckets) return;
@@ -25,7 +26,7 @@ __global__ void __launch_bounds__(32 * kSolveWarpsPerBlock)
   double* G = Gs[wi];
   double* beta = Bs[wi];
   reduce_bucket(v, b, G, lane);
-  const int st = solve_bucket_warp(K, G, p, b, beta, lane);
+  const int st = solve_bucket_warp(K, G, Fs[wi], p, b, beta, lane);
   for (int k = lane; k < K; k += 32) {
     const float f = (float)beta[k];
     v.beta[b * K + k] = f;

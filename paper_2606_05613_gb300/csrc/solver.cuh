@@ -27,8 +27,8 @@
 //    one lane per task.
 //  MEAN: beta = 1/K.
 //
-// All solvers work on G scaled so that max_k G_kk = 1 (every rule is
-// invariant under a positive scaling of G).  A Gram with a NaN or Inf gives
+// All solvers work on G scaled by a power of two so that max_k G_kk lies in
+// [1, 2) (every rule is invariant under a positive scaling of G).  A Gram with a NaN or Inf gives
 // beta = 1/K and status BKMOO_ERR_NONFINITE.
 #pragma once
 
@@ -650,7 +650,7 @@ __device__ __forceinline__ bool in_mask(unsigned m, int k) {
 // K + 1).  Returns its squared norm in fp32, +inf if S is singular or the
 // point leaves the simplex; Ainv and z for the refinement.
 template <int K>
-__device__ float mgda_candidate32(const double* G, unsigned mask, float (&Ainv)[K + 1][K + 1],
+__device__ float mgda_candidate32(const float* G, unsigned mask, float (&Ainv)[K + 1][K + 1],
                                   float (&z)[K + 1]) {
   constexpr int N = K + 1;
   float A[N][N];
@@ -658,7 +658,7 @@ __device__ float mgda_candidate32(const double* G, unsigned mask, float (&Ainv)[
   for (int i = 0; i < K; ++i) {
 #pragma unroll
     for (int j = 0; j < K; ++j)
-      A[i][j] = (in_mask<K>(mask, i) && in_mask<K>(mask, j)) ? (float)G[i * K + j]
+      A[i][j] = (in_mask<K>(mask, i) && in_mask<K>(mask, j)) ? G[i * K + j]
                 : (i == j && !in_mask<K>(mask, i)) ? 1.0f : 0.0f;
     A[i][K] = in_mask<K>(mask, i) ? 1.0f : 0.0f;
     A[K][i] = in_mask<K>(mask, i) ? 1.0f : 0.0f;
@@ -675,14 +675,14 @@ __device__ float mgda_candidate32(const double* G, unsigned mask, float (&Ainv)[
     if (z[i] < -1e-5f) ok = false;
 #pragma unroll
     for (int j = 0; j < K; ++j)
-      if (in_mask<K>(mask, j)) q = fmaf(z[i] * (float)G[i * K + j], z[j], q);
+      if (in_mask<K>(mask, j)) q = fmaf(z[i] * G[i * K + j], z[j], q);
   }
   return ok ? q : INFINITY;
 }
 
-// Two mixed-precision refinement steps of A z = e_K in fp64 (residual in
-// fp64, correction through the fp32 inverse), then alpha = z on S, >= 0,
-// renormalised.
+// One mixed-precision refinement step of A z = e_K (residual in fp64,
+// correction through the fp32 inverse: error about (cond(A) 2^-24)^2), then
+// alpha = z on S, >= 0, renormalised.
 template <int K>
 __device__ void mgda_refine(const double* G, unsigned mask, const float (&Ainv)[K + 1][K + 1],
                             const float (&z32)[K + 1], double (&alpha)[K]) {
@@ -690,8 +690,7 @@ __device__ void mgda_refine(const double* G, unsigned mask, const float (&Ainv)[
   double z[N];
 #pragma unroll
   for (int i = 0; i < N; ++i) z[i] = z32[i];
-#pragma unroll
-  for (int it = 0; it < 2; ++it) {
+  {
     float r[N];
 #pragma unroll
     for (int i = 0; i < K; ++i) {
@@ -733,12 +732,12 @@ __device__ void mgda_refine(const double* G, unsigned mask, const float (&Ainv)[
 // Exact MGDA for 2 <= K <= 5.  False (beta untouched) if the optimality
 // check fails; the caller then takes the serial fp64 path.
 template <int K>
-__device__ bool mgda_fast(const double* G, int lane, double* beta_out) {
+__device__ bool mgda_fast(const double* G, const float* Gf, int lane, double* beta_out) {
   constexpr int N = K + 1;
   float Ainv[N][N], z[N];
   const unsigned mask = (unsigned)lane + 1u;
   float q = INFINITY;
-  if (mask < (1u << K)) q = mgda_candidate32<K>(G, mask, Ainv, z);
+  if (mask < (1u << K)) q = mgda_candidate32<K>(Gf, mask, Ainv, z);
   const int win = warp_argmin(q, lane);
   const unsigned wmask = (unsigned)win + 1u;
   double alpha[K];
@@ -746,21 +745,42 @@ __device__ bool mgda_fast(const double* G, int lane, double* beta_out) {
 #pragma unroll
   for (int k = 0; k < K; ++k) alpha[k] = __shfl_sync(0xffffffffu, alpha[k], win);
   if (!(__shfl_sync(0xffffffffu, q, win) < INFINITY)) return false;
-  // optimality: <g_k, d> >= ||d||^2 for every k (proof of Theorem 3.1)
-  double v[K], xx = 0.0, vmin = 1e300;
+  // optimality: <g_k, d> >= ||d||^2 for every k (proof of Theorem 3.1); on
+  // S it holds with equality by construction, off S it is checked in fp32
+  // with a margin far above fp32 rounding, and in fp64 only when marginal
+  {
+    float a32[K], v32[K], xx32 = 0.0f;
 #pragma unroll
-  for (int k = 0; k < K; ++k) {
-    double t = 0.0;
+    for (int k = 0; k < K; ++k) a32[k] = (float)alpha[k];
 #pragma unroll
-    for (int j = 0; j < K; ++j) t = fma(G[k * K + j], alpha[j], t);
-    v[k] = t;
+    for (int k = 0; k < K; ++k) {
+      float t = 0.0f;
+#pragma unroll
+      for (int j = 0; j < K; ++j) t = fmaf(Gf[k * K + j], a32[j], t);
+      v32[k] = t;
+      xx32 = fmaf(a32[k], t, xx32);
+    }
+    bool clear = true;
+#pragma unroll
+    for (int k = 0; k < K; ++k)
+      if (!in_mask<K>(wmask, k) && !(v32[k] - xx32 >= 1e-5f)) clear = false;
+    if (!clear) {
+      double v[K], xx = 0.0, vmin = 1e300;
+#pragma unroll
+      for (int k = 0; k < K; ++k) {
+        double t = 0.0;
+#pragma unroll
+        for (int j = 0; j < K; ++j) t = fma(G[k * K + j], alpha[j], t);
+        v[k] = t;
+      }
+#pragma unroll
+      for (int k = 0; k < K; ++k) {
+        xx = fma(alpha[k], v[k], xx);
+        vmin = fmin(vmin, v[k]);
+      }
+      if (!(vmin >= xx - kKkt)) return false;
+    }
   }
-#pragma unroll
-  for (int k = 0; k < K; ++k) {
-    xx = fma(alpha[k], v[k], xx);
-    vmin = fmin(vmin, v[k]);
-  }
-  if (!(vmin >= xx - kKkt)) return false;
   if (lane == 0)
 #pragma unroll
     for (int k = 0; k < K; ++k) beta_out[k] = alpha[k];
@@ -772,7 +792,7 @@ __device__ bool mgda_fast(const double* G, int lane, double* beta_out) {
 // cag_affine), F there (+inf if S is singular, D <= 0 or w leaves the
 // simplex); the fp32 inverse of the masked G_SS for the refinement.
 template <int K>
-__device__ float cagrad_candidate32(const double* G, const float (&b)[K], float rho,
+__device__ float cagrad_candidate32(const float* G, const float (&b)[K], float rho,
                                     unsigned mask, float (&Ginv)[K][K], float (&w)[K]) {
   const int s = __popc(mask);
 #pragma unroll
@@ -784,7 +804,7 @@ __device__ float cagrad_candidate32(const double* G, const float (&b)[K], float 
     for (int k = 0; k < K; ++k)
       if (k == k0) {
         w[k] = 1.0f;
-        gkk = (float)G[k * K + k];
+        gkk = G[k * K + k];
         bk = b[k];
       }
     return bk + rho * sqrtf(fmaxf(gkk, 0.0f));
@@ -794,7 +814,7 @@ __device__ float cagrad_candidate32(const double* G, const float (&b)[K], float 
   for (int i = 0; i < K; ++i)
 #pragma unroll
     for (int j = 0; j < K; ++j)
-      A[i][j] = (in_mask<K>(mask, i) && in_mask<K>(mask, j)) ? (float)G[i * K + j]
+      A[i][j] = (in_mask<K>(mask, i) && in_mask<K>(mask, j)) ? G[i * K + j]
                 : (i == j && !in_mask<K>(mask, i)) ? 1.0f : 0.0f;
   if (!inverse32<K>(A, Ginv, 1e-6f)) return INFINITY;
   float om = 0.0f, on = 0.0f, nb = 0.0f, m[K], n[K];
@@ -837,12 +857,12 @@ __device__ float cagrad_candidate32(const double* G, const float (&b)[K], float 
 #pragma unroll
   for (int i = 0; i < K; ++i)
 #pragma unroll
-    for (int j = 0; j < K; ++j) q = fmaf(w[i] * (float)G[i * K + j], w[j], q);
+    for (int j = 0; j < K; ++j) q = fmaf(w[i] * G[i * K + j], w[j], q);
   return bw + rho * sqrtf(fmaxf(q, 0.0f));
 }
 
 // fp64 stationary point on the winning support: m = G_SS^-1 1 and
-// n = G_SS^-1 b_S refined twice, then the closed form.
+// n = G_SS^-1 b_S with one refinement step, then the closed form.
 template <int K>
 __device__ void cagrad_refine(const double* G, const double (&b)[K], double rho, unsigned mask,
                               const float (&Ginv)[K][K], double (&w)[K]) {
@@ -864,8 +884,7 @@ __device__ void cagrad_refine(const double* G, const double (&b)[K], double rho,
     m[i] = mi;
     n[i] = ni;
   }
-#pragma unroll
-  for (int it = 0; it < 2; ++it) {
+  {
     float rm[K], rn[K];
 #pragma unroll
     for (int i = 0; i < K; ++i) {
@@ -924,7 +943,8 @@ __device__ void cagrad_refine(const double* G, const double (&b)[K], double rho,
 // Exact CAGrad for 1 <= K <= 5.  False if the check fails or a case that
 // needs the minimum-norm candidate (0 possibly in the hull) comes up.
 template <int K>
-__device__ bool cagrad_fast(const double* G, double c, int lane, double* beta_out) {
+__device__ bool cagrad_fast(const double* G, const float* Gf, double c, int lane,
+                            double* beta_out) {
   double b[K], tot = 0.0;
   float bf[K];
 #pragma unroll
@@ -951,7 +971,7 @@ __device__ bool cagrad_fast(const double* G, double c, int lane, double* beta_ou
   float Ginv[K][K], w32[K];
   const unsigned mask = (unsigned)lane + 1u;
   float F = INFINITY;
-  if (mask < (1u << K)) F = cagrad_candidate32<K>(G, bf, (float)rho, mask, Ginv, w32);
+  if (mask < (1u << K)) F = cagrad_candidate32<K>(Gf, bf, (float)rho, mask, Ginv, w32);
   const int win = warp_argmin(F, lane);
   if (!(__shfl_sync(0xffffffffu, F, win) < INFINITY)) return false;
   double w[K];
@@ -959,25 +979,66 @@ __device__ bool cagrad_fast(const double* G, double c, int lane, double* beta_ou
 #pragma unroll
   for (int k = 0; k < K; ++k) w[k] = __shfl_sync(0xffffffffu, w[k], win);
   // optimality of the dual: grad_k = b_k + rho (G w)_k / ||g_w|| >= w^T grad
+  // (equality on the support); fp32 with a margin, fp64 when marginal
+  const unsigned wmask = (unsigned)win + 1u;
   double v[K], q = 0.0;
+#pragma unroll
+  for (int k = 0; k < K; ++k) {
+    float t = 0.0f;
+#pragma unroll
+    for (int j = 0; j < K; ++j) t = fmaf(Gf[k * K + j], (float)w[j], t);
+    v[k] = t;
+  }
+  {
+    float q32 = 0.0f;
+#pragma unroll
+    for (int k = 0; k < K; ++k) q32 = fmaf((float)w[k], (float)v[k], q32);
+    if (!(q32 > 1e-12f)) return false;
+    const float f32 = (float)rho / sqrtf(q32);
+    float lam32 = 0.0f;
+    float g32[K];
+#pragma unroll
+    for (int k = 0; k < K; ++k) {
+      g32[k] = fmaf(f32, (float)v[k], bf[k]);
+      lam32 = fmaf((float)w[k], g32[k], lam32);
+    }
+    bool clear = true;
+#pragma unroll
+    for (int k = 0; k < K; ++k)
+      if (!in_mask<K>(wmask, k) && !(g32[k] - lam32 >= 1e-5f)) clear = false;
+    if (!clear) {
+#pragma unroll
+      for (int k = 0; k < K; ++k) {
+        double t = 0.0;
+#pragma unroll
+        for (int j = 0; j < K; ++j) t = fma(G[k * K + j], w[j], t);
+        v[k] = t;
+      }
+      double qq = 0.0;
+#pragma unroll
+      for (int k = 0; k < K; ++k) qq = fma(w[k], v[k], qq);
+      if (!(qq > 1e-24)) return false;
+      const double fd = div_nr(rho, sqrt_nr(qq));
+      double lam = 0.0, gmin = 1e300;
+#pragma unroll
+      for (int k = 0; k < K; ++k) {
+        const double gk = fma(fd, v[k], b[k]);
+        lam = fma(w[k], gk, lam);
+        gmin = fmin(gmin, gk);
+      }
+      if (!(gmin >= lam - 1e-11)) return false;
+    }
+  }
+  // beta = 1/K + rho w / ||g_w|| with ||g_w|| in fp64
 #pragma unroll
   for (int k = 0; k < K; ++k) {
     double t = 0.0;
 #pragma unroll
     for (int j = 0; j < K; ++j) t = fma(G[k * K + j], w[j], t);
-    v[k] = t;
     q = fma(w[k], t, q);
   }
   if (!(q > 1e-24)) return false;
   const double f = div_nr(rho, sqrt_nr(q));
-  double lam = 0.0, gmin = 1e300;
-#pragma unroll
-  for (int k = 0; k < K; ++k) {
-    const double gk = fma(f, v[k], b[k]);
-    lam = fma(w[k], gk, lam);
-    gmin = fmin(gmin, gk);
-  }
-  if (!(gmin >= lam - 1e-11)) return false;
   if (lane == 0)
 #pragma unroll
     for (int k = 0; k < K; ++k) beta_out[k] = fma(f, w[k], 1.0 / K);
@@ -1026,8 +1087,8 @@ __device__ void pcgrad_fast(const double* G, uint64_t seed, uint64_t step, int64
 }
 
 template <int K>
-__device__ bool solve_fast_k(int rule, const double* G, const SolveParams& p, int64_t b,
-                             int lane, double* beta_out) {
+__device__ bool solve_fast_k(int rule, const double* G, const float* Gf, const SolveParams& p,
+                             int64_t b, int lane, double* beta_out) {
   if (rule == BKMOO_PCGRAD) {
     pcgrad_fast<K>(G, p.seed, p.step, b, lane, beta_out);
     return true;
@@ -1035,19 +1096,20 @@ __device__ bool solve_fast_k(int rule, const double* G, const SolveParams& p, in
   if (K > kEnumMaxK || !(p.flags & BKMOO_FLAG_POLISH)) return false;
   if (rule == BKMOO_MGDA) {
     if (K < 2 || (K == 2 && (p.flags & BKMOO_FLAG_CLOSED_FORM_K2))) return false;
-    return mgda_fast<(K <= kEnumMaxK ? K : 2)>(G, lane, beta_out);
+    return mgda_fast<(K <= kEnumMaxK ? K : 2)>(G, Gf, lane, beta_out);
   }
-  if (rule == BKMOO_CAGRAD) return cagrad_fast<(K <= kEnumMaxK ? K : 1)>(G, p.cagrad_c, lane, beta_out);
+  if (rule == BKMOO_CAGRAD)
+    return cagrad_fast<(K <= kEnumMaxK ? K : 1)>(G, Gf, p.cagrad_c, lane, beta_out);
   return false;
 }
 
 // Dispatch on K; true when a fast path produced beta (valid on every lane
 // after the caller's __syncwarp).
-__device__ bool solve_fast(int K, int rule, const double* G, const SolveParams& p, int64_t b,
-                           int lane, double* beta_out) {
+__device__ bool solve_fast(int K, int rule, const double* G, const float* Gf,
+                           const SolveParams& p, int64_t b, int lane, double* beta_out) {
   switch (K) {
 #define BKMOO_FAST_CASE(k) \
-  case k: return solve_fast_k<k>(rule, G, p, b, lane, beta_out);
+  case k: return solve_fast_k<k>(rule, G, Gf, p, b, lane, beta_out);
     BKMOO_FAST_CASE(1) BKMOO_FAST_CASE(2) BKMOO_FAST_CASE(3) BKMOO_FAST_CASE(4)
     BKMOO_FAST_CASE(5) BKMOO_FAST_CASE(6) BKMOO_FAST_CASE(7) BKMOO_FAST_CASE(8)
     BKMOO_FAST_CASE(9) BKMOO_FAST_CASE(10) BKMOO_FAST_CASE(11) BKMOO_FAST_CASE(12)
@@ -1064,33 +1126,54 @@ __device__ bool solve_fast(int K, int rule, const double* G, const SolveParams& 
 // The whole warp enters with G (K x K) in shared memory; G is normalised in
 // place.  beta_out (shared, K entries) and the returned status are valid on
 // every lane after the call.
-__device__ int solve_bucket_warp(int K, double* G, const SolveParams& p, int64_t b,
+__device__ int solve_bucket_warp(int K, double* G, float* Gf, const SolveParams& p, int64_t b,
                                  double* beta_out, int lane) {
+  // finiteness and the largest diagonal entry from the bit patterns
+  // (non-negative doubles order as integers), then an exact power-of-two
+  // scaling that brings max_k G_kk into [1, 2)
   bool finite = true;
-  double scale = 0.0;
-  for (int i = 0; i < K * K; ++i)
-    if (!isfinite(G[i])) finite = false;
-  for (int k = 0; k < K; ++k) scale = fmax(scale, G[k * K + k]);
-  __syncwarp();
+  long long dmax = 0;
+  for (int i = lane; i < K * K; i += 32) {
+    const long long bits = __double_as_longlong(G[i]);
+    if (((bits >> 52) & 0x7ff) == 0x7ff) finite = false;
+    if (i / K == i % K && bits > dmax) dmax = bits;
+  }
+  finite = __all_sync(0xffffffffu, finite);
+  for (int off = 16; off > 0; off >>= 1) {
+    const long long o = __shfl_xor_sync(0xffffffffu, dmax, off);
+    dmax = o > dmax ? o : dmax;
+  }
   if (!finite) {
     if (lane == 0)
       for (int k = 0; k < K; ++k) beta_out[k] = 1.0 / K;
     __syncwarp();
     return BKMOO_ERR_NONFINITE;
   }
-  if (scale > 0.0) {
-    const double inv = 1.0 / scale;
-    for (int i = lane; i < K * K; i += 32) G[i] *= inv;
+  double top = 1.0;
+  if (dmax > 0) {
+    const int e = (int)((dmax >> 52) & 0x7ff) - 1023;
+    if (e > -1022 && e < 1023) {
+      const double f = __longlong_as_double((long long)(1023 - e) << 52);
+      for (int i = lane; i < K * K; i += 32) G[i] *= f;
+      top = __longlong_as_double(dmax) * f;
+    } else {  // extreme scales: plain division
+      const double inv = 1.0 / __longlong_as_double(dmax);
+      for (int i = lane; i < K * K; i += 32) G[i] *= inv;
+    }
   }
   __syncwarp();
+  for (int i = lane; i < K * K; i += 32) Gf[i] = (float)G[i];
+  __syncwarp();
+  SolveParams q = p;
+  q.tol = p.tol * top;  // the stopping test is relative to max_k G_kk
   int st = BKMOO_OK;
-  const bool fast = solve_fast(K, p.rule, G, p, b, lane, beta_out);
+  const bool fast = solve_fast(K, q.rule, G, Gf, q, b, lane, beta_out);
   if (!fast && lane == 0) {
     double beta[kMaxK];
-    switch (p.rule) {
-      case BKMOO_MGDA: st = solve_mgda(K, G, p, beta); break;
-      case BKMOO_PCGRAD: st = solve_pcgrad(K, G, p, b, beta); break;
-      case BKMOO_CAGRAD: st = solve_cagrad(K, G, p, beta); break;
+    switch (q.rule) {
+      case BKMOO_MGDA: st = solve_mgda(K, G, q, beta); break;
+      case BKMOO_PCGRAD: st = solve_pcgrad(K, G, q, b, beta); break;
+      case BKMOO_CAGRAD: st = solve_cagrad(K, G, q, beta); break;
       default:
         for (int k = 0; k < K; ++k) beta[k] = 1.0 / K;
     }
