@@ -155,6 +155,23 @@ int bkmoo_gram(const void* const* grads, int32_t K, int32_t in_dtype,
                void* ws, size_t ws_bytes, void* stream);
 
 /*
+ * bkmoo_conflicts -- the gradient-conflict statistics of Figure 1, per
+ * bucket, from Gram matrices (bkmoo_gram's out_gram): the pairwise cosines
+ * cos_ij = G_ij / sqrt(G_ii G_jj) -- a pair conflicts when its cosine is
+ * negative (Eq. 2, Definition A.4) -- their mean, population standard
+ * deviation and minimum over the K(K-1)/2 pairs, and a flag for "at least
+ * one pair conflicts" (the event whose per-layer frequency over training
+ * steps Figure 1 plots).  A pair with a zero-norm gradient has cosine 0.
+ *
+ * gram: device fp64 [n_buckets][K][K].  Outputs (device, each may be NULL):
+ * out_cos fp32 [n_buckets][K][K] (diagonal 1, or 0 for a zero gradient),
+ * out_stats fp32 [n_buckets][3] = (mean, std, min), out_conflict int32
+ * [n_buckets] in {0, 1}.  2 <= K <= 16, else BKMOO_ERR_INVALID.
+ */
+int bkmoo_conflicts(const double* gram, int32_t K, int64_t n_buckets, float* out_cos,
+                    float* out_stats, int32_t* out_conflict, void* stream);
+
+/*
  * bkmoo_gram_noalloc -- bkmoo_gram without a workspace argument; it allocates
  * no memory at all.  The paper has no counterpart: this is a service for
  * callers that hold their input and output buffers but cannot get more

@@ -668,6 +668,47 @@ void bko_combine(int32_t K, int32_t dtype, const void* const* x,
 }
 
 /* ------------------------------------------------------------------------ */
+/* Conflict statistics of Figure 1 (Eq. 2, Definition A.4).                  */
+/* ------------------------------------------------------------------------ */
+
+/*
+ * Pairwise cosines cos_ij = G_ij / sqrt(G_ii G_jj) (0 when either gradient is
+ * zero; 1 on the diagonal of a non-zero gradient); over the K(K-1)/2 pairs
+ * i < j: mean, population standard deviation (the square root of the mean
+ * squared deviation from the mean), minimum; conflict = 1 when some pair has
+ * a negative cosine.  cos (K*K) may be NULL.  stats = (mean, std, min).
+ */
+void bko_conflicts(int32_t K, const double* G, double* cos, double* stats,
+                   int32_t* conflict) {
+  double c[KMAX * KMAX];
+  int32_t any = 0;
+  double sum = 0.0, mn = 1.0;
+  int np = 0;
+  for (int i = 0; i < K; ++i)
+    for (int j = 0; j < K; ++j) {
+      double gi = G[i * K + i], gj = G[j * K + j];
+      double v;
+      if (i == j) v = gi > 0.0 ? 1.0 : 0.0;
+      else v = (gi > 0.0 && gj > 0.0) ? G[i * K + j] / sqrt(gi * gj) : 0.0;
+      c[i * K + j] = v;
+      if (i < j) {
+        sum += v;
+        ++np;
+        if (v < mn) mn = v;
+        if (v < 0.0) any = 1;
+      }
+    }
+  double mean = np ? sum / np : 0.0, dev = 0.0;
+  for (int i = 0; i < K; ++i)
+    for (int j = i + 1; j < K; ++j) dev += (c[i * K + j] - mean) * (c[i * K + j] - mean);
+  stats[0] = mean;
+  stats[1] = np ? sqrt(dev / np) : 0.0;
+  stats[2] = mn;
+  if (cos) memcpy(cos, c, sizeof(double) * K * K);
+  *conflict = any;
+}
+
+/* ------------------------------------------------------------------------ */
 /* Whole path over buckets [b0, b1): Gram -> rule -> combination.            */
 /* ------------------------------------------------------------------------ */
 

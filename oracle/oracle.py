@@ -86,6 +86,8 @@ def _load():
         lib.bko_pcgrad.argtypes = [i32, vp, u64, u64, i64, vp, vp]
         lib.bko_cagrad.restype = None
         lib.bko_cagrad.argtypes = [i32, vp, dbl, vp, vp]
+        lib.bko_conflicts.restype = None
+        lib.bko_conflicts.argtypes = [i32, vp, vp, vp, vp]
         lib.bko_combine.restype = None
         lib.bko_combine.argtypes = [i32, i32, vp, i64, i64, vp, vp]
         lib.bko_resolve.restype = ctypes.c_int
@@ -205,6 +207,17 @@ def cagrad(G, c: float):
     w = np.zeros(K)
     _load().bko_cagrad(K, _ptr(G), c, _ptr(b), _ptr(w))
     return b, w
+
+
+def conflicts(G):
+    """Figure 1 statistics of one bucket: (cos matrix, (mean, std, min), conflict flag)."""
+    G = _as_G(G)
+    K = G.shape[0]
+    cos = np.zeros((K, K))
+    stats = np.zeros(3)
+    flag = np.zeros(1, dtype=np.int32)
+    _load().bko_conflicts(K, _ptr(G), _ptr(cos), _ptr(stats), _ptr(flag))
+    return cos, stats, int(flag[0])
 
 
 def combine(xs, beta, begin: int = 0, n: int | None = None) -> np.ndarray:

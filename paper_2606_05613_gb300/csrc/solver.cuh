@@ -9,9 +9,13 @@
 //      lane: lane l takes S = the bits of l + 1, finds the affine
 //      minimum-norm point of S in fp32 and keeps it if it lies in the
 //      simplex; the least norm wins, is refined in fp64 and checked.
-//    Otherwise Frank-Wolfe from the best pair with exact line search (lane
-//      0), then (POLISH) an exact active-set completion in the manner of
-//      Wolfe's minimum-norm-point algorithm: the affine minimum-norm point of
+//    K >= 6 with POLISH: Wolfe's minimum-norm-point algorithm in fp32 with a
+//      lane-parallel Gauss-Jordan, one fp64 refinement of the final support
+//      and the same check.
+//    Without POLISH, or when a check fails: Frank-Wolfe from the best pair
+//      with exact line search (lane 0, fp64), then (POLISH) an exact
+//      active-set completion in the manner of Wolfe's minimum-norm-point
+//      algorithm: the affine minimum-norm point of
 //      the current support is taken when it lies inside the simplex, else the
 //      iterate moves to the boundary and drops a point; a point is added
 //      while some g_j has <d, g_j> < ||d||^2.
@@ -20,8 +24,12 @@
 //    K <= 5 with POLISH: exact, one support per lane, with the closed-form
 //      stationary point of F on the support's affine hull (fp32 search,
 //      fp64 refinement and check).
-//    Otherwise Frank-Wolfe with exact line search from the best vertex (lane
-//      0), then (POLISH) the same kind of active-set completion.
+//    K >= 6 with POLISH: the same kind of active-set method in fp32 with the
+//      lane-parallel Gauss-Jordan, from the best vertex; fp64 refinement and
+//      check.
+//    Without POLISH, or when a check fails: Frank-Wolfe with exact line
+//      search from the best vertex (lane 0, fp64), then (POLISH) the same
+//      kind of active-set completion.
 //  PCGrad (Eq. 5; Eq. 8): the projections of Algorithm 1 carried out on the
 //    coefficients of each running d_t, since <d_t, g_j> = sum_m C_tm G_mj;
 //    one lane per task.
@@ -1086,6 +1094,350 @@ __device__ void pcgrad_fast(const double* G, uint64_t seed, uint64_t step, int64
   }
 }
 
+// ---------------------------------------------------------------------------
+// K >= 6: Wolfe's algorithm in fp32 with a lane-parallel Gauss-Jordan
+// ---------------------------------------------------------------------------
+
+constexpr int kUnk = kMaxK + 1;   // up to kMaxK + 1 unknowns
+constexpr int kCols = kUnk + 2;   // two right-hand sides in slots kUnk, kUnk + 1
+
+// Position of the n-th (0-based) set bit of m.
+__device__ __forceinline__ int nth_set(unsigned m, int n) {
+  for (int i = 0; i < n; ++i) m &= m - 1u;
+  return __ffs(m) - 1;
+}
+
+__device__ __forceinline__ int warp_argmin_f(float val, int lane) { return warp_argmin(val, lane); }
+
+__device__ __forceinline__ float warp_sum_f(float x) {
+  for (int off = 16; off > 0; off >>= 1) x += __shfl_xor_sync(0xffffffffu, x, off);
+  return x;
+}
+
+// Lane i < m holds row i of an m-unknown system: coefficients in row[0..m-1]
+// (slots m .. kUnk-1 are zero) and two right-hand sides in row[kUnk] and
+// row[kUnk + 1].  Gauss-Jordan with partial pivoting across lanes;
+// afterwards lane i < m holds the two solutions' i-th entries in the same
+// slots.  False when a pivot is below `piv`.
+__device__ bool warp_gauss_jordan(float (&row)[kCols], int m, int lane, float piv) {
+  bool ok = true;
+#pragma unroll
+  for (int c = 0; c < kUnk; ++c) {
+    if (c >= m) break;
+    float a = (lane >= c && lane < m) ? fabsf(row[c]) : -1.0f;
+    int p = lane;
+    for (int off = 16; off > 0; off >>= 1) {
+      const float a2 = __shfl_xor_sync(0xffffffffu, a, off);
+      const int p2 = __shfl_xor_sync(0xffffffffu, p, off);
+      if (a2 > a || (a2 == a && p2 < p)) {
+        a = a2;
+        p = p2;
+      }
+    }
+    if (!(a > piv)) ok = false;
+    const int src = lane == c ? p : (lane == p ? c : lane);
+#pragma unroll
+    for (int j = c; j < kCols; ++j) row[j] = __shfl_sync(0xffffffffu, row[j], src);
+    const float inv = __frcp_rn(__shfl_sync(0xffffffffu, row[c], c));
+    const float f = row[c];
+#pragma unroll
+    for (int j = c; j < kCols; ++j) {
+      const float pj = __shfl_sync(0xffffffffu, row[j], c) * inv;
+      if (lane == c) row[j] = pj;
+      else if (lane < m) row[j] = fmaf(-f, pj, row[j]);
+    }
+  }
+  return ok;
+}
+
+// Bordered system of the affine minimum-norm point of support smask
+// (s = |S| rows of G_SS | 1, then the row 1^T | 0); rhs supplied per lane.
+__device__ __forceinline__ void mgda_rows(const float* Gf, int K, unsigned smask, int lane,
+                                          float rhs, float (&row)[kCols]) {
+  const int s = __popc(smask);
+  const int pi = lane < s ? nth_set(smask, lane) : 0;
+#pragma unroll
+  for (int j = 0; j < kUnk; ++j) {
+    float v = 0.0f;
+    if (j < s) {
+      const int pj = nth_set(smask, j);
+      v = lane < s ? Gf[pi * K + pj] : (lane == s ? 1.0f : 0.0f);
+    } else if (j == s) {
+      v = lane < s ? 1.0f : 0.0f;
+    }
+    row[j] = v;
+  }
+  row[kUnk] = rhs;
+  row[kUnk + 1] = 0.0f;
+}
+
+// Exact MGDA for any K (used for K >= 6): Wolfe's minimum-norm-point method
+// on the fp32 Gram with lane k holding weight lam_k, then one fp64
+// refinement of the final support and the optimality check.  False (beta
+// untouched) if a system is singular or the check fails.
+__device__ bool mgda_wolfe_warp(int K, const double* G, const float* Gf, int lane,
+                                double* beta_out) {
+  const bool act = lane < K;
+  const int k0 = warp_argmin_f(act ? Gf[lane * K + lane] : INFINITY, lane);
+  bool in = lane == k0;
+  float lam = in ? 1.0f : 0.0f;
+  float row[kCols];
+  for (int major = 0; major < 4 * K + 4; ++major) {
+    float v = 0.0f;
+    for (int j = 0; j < K; ++j) {
+      const float lj = __shfl_sync(0xffffffffu, lam, j);
+      if (act) v = fmaf(Gf[lane * K + j], lj, v);
+    }
+    const float xx = warp_sum_f(act ? lam * v : 0.0f);
+    const int jn = warp_argmin_f(act ? v : INFINITY, lane);
+    const float vj = __shfl_sync(0xffffffffu, v, jn);
+    if (vj >= xx - 1e-6f) break;
+    if (__shfl_sync(0xffffffffu, in ? 1 : 0, jn)) break;
+    if (lane == jn) {
+      in = true;
+      lam = 0.0f;
+    }
+    bool settled = false;
+    for (int minor = 0; minor <= K + 1 && !settled; ++minor) {
+      const unsigned smask = __ballot_sync(0xffffffffu, in && act);
+      const int s = __popc(smask);
+      if (s == 0) return false;
+      mgda_rows(Gf, K, smask, lane, lane == s ? 1.0f : 0.0f, row);
+      if (!warp_gauss_jordan(row, s + 1, lane, 1e-6f)) return false;
+      const int rank = __popc(smask & ((1u << lane) - 1u));
+      const float mu_all = __shfl_sync(0xffffffffu, row[kUnk], in ? rank : 0);
+      const float mu = in ? mu_all : 0.0f;
+      if (__all_sync(0xffffffffu, !in || mu > 1e-7f)) {
+        lam = mu;
+        settled = true;
+        break;
+      }
+      const float t = (in && mu <= 1e-7f) ? ((lam - mu) > 0.0f ? lam / (lam - mu) : 0.0f)
+                                          : INFINITY;
+      const int drop = warp_argmin_f(t, lane);
+      const float theta = __shfl_sync(0xffffffffu, t, drop);
+      lam = in ? (1.0f - theta) * lam + theta * mu : 0.0f;
+      if (lane == drop || lam <= 1e-7f) {
+        in = false;
+        lam = 0.0f;
+      }
+    }
+    if (!settled) return false;
+  }
+  // one fp64 refinement of the final support's bordered system
+  const unsigned smask = __ballot_sync(0xffffffffu, in && act);
+  const int s = __popc(smask);
+  if (s == 0) return false;
+  mgda_rows(Gf, K, smask, lane, lane == s ? 1.0f : 0.0f, row);
+  if (!warp_gauss_jordan(row, s + 1, lane, 1e-6f)) return false;
+  double z = (lane <= s) ? (double)row[kUnk] : 0.0;   // lane i <= s: unknown i
+  double r = 0.0;
+  {
+    const int pi = lane < s ? nth_set(smask, lane) : 0;
+    double acc = 0.0;
+    for (int j = 0; j <= s; ++j) {
+      const double zj = __shfl_sync(0xffffffffu, z, j);
+      if (lane < s) {
+        const double a = j < s ? G[pi * K + nth_set(smask, j)] : 1.0;
+        acc = fma(a, zj, acc);
+      } else if (lane == s && j < s) {
+        acc += zj;
+      }
+    }
+    r = lane < s ? -acc : (lane == s ? 1.0 - acc : 0.0);
+  }
+  mgda_rows(Gf, K, smask, lane, (float)r, row);
+  if (!warp_gauss_jordan(row, s + 1, lane, 1e-6f)) return false;
+  z += (lane <= s) ? (double)row[kUnk] : 0.0;
+  // alpha on lanes k < K
+  const int rank = __popc(smask & ((1u << lane) - 1u));
+  const bool ink = act && ((smask >> lane) & 1u);
+  const double zk = __shfl_sync(0xffffffffu, z, ink ? rank : 0);
+  double alpha = (ink && zk > 0.0) ? zk : 0.0;
+  double sum = alpha;
+  for (int off = 16; off > 0; off >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, off);
+  alpha *= (2.0 - sum);
+  // optimality (proof of Theorem 3.1): fp32 with a margin, fp64 if marginal
+  const float a32 = (float)alpha;
+  float v32 = 0.0f;
+  for (int j = 0; j < K; ++j) {
+    const float aj = __shfl_sync(0xffffffffu, a32, j);
+    if (act) v32 = fmaf(Gf[lane * K + j], aj, v32);
+  }
+  const float xx32 = warp_sum_f(act ? a32 * v32 : 0.0f);
+  const bool clear = !act || ink || (v32 - xx32 >= 1e-5f);
+  if (!__all_sync(0xffffffffu, clear)) {
+    double v = 0.0;
+    for (int j = 0; j < K; ++j) {
+      const double aj = __shfl_sync(0xffffffffu, alpha, j);
+      if (act) v = fma(G[lane * K + j], aj, v);
+    }
+    double xx = act ? alpha * v : 0.0;
+    for (int off = 16; off > 0; off >>= 1) xx += __shfl_xor_sync(0xffffffffu, xx, off);
+    if (!__all_sync(0xffffffffu, !act || v >= xx - kKkt)) return false;
+  }
+  if (act) beta_out[lane] = alpha;
+  return true;
+}
+
+// Rows of G_SS [m n] = [1 b_S] for support smask (lane i < s: row i).
+__device__ __forceinline__ void cagrad_rows(const float* Gf, int K, unsigned smask, int lane,
+                                            float bi, float r1, float r2, float (&row)[kCols]) {
+  const int s = __popc(smask);
+  const int pi = lane < s ? nth_set(smask, lane) : 0;
+#pragma unroll
+  for (int j = 0; j < kUnk; ++j)
+    row[j] = (j < s && lane < s) ? Gf[pi * K + nth_set(smask, j)] : 0.0f;
+  row[kUnk] = lane < s ? r1 : 0.0f;
+  row[kUnk + 1] = lane < s ? r2 : 0.0f;
+  (void)bi;
+}
+
+// Exact CAGrad for any K (used for K >= 6): active-set method on the dual
+// min_{w in simplex} b^T w + rho ||g_w|| from the best vertex, with the
+// closed-form stationary point of each support (see cag_affine) solved by
+// the lane-parallel Gauss-Jordan in fp32; then m, n refined once in fp64,
+// the closed form in fp64 and the optimality check.  Lane k holds w_k.
+__device__ bool cagrad_active_warp(int K, const double* G, const float* Gf, double c, int lane,
+                                   double* beta_out) {
+  const bool act = lane < K;
+  // b_k = <g_k, g0>, ||g0||^2 (fp64 for the final coefficients)
+  double bd = 0.0;
+  if (act)
+    for (int j = 0; j < K; ++j) bd += G[lane * K + j];
+  double tot = bd;
+  for (int off = 16; off > 0; off >>= 1) tot += __shfl_xor_sync(0xffffffffu, tot, off);
+  bd *= 1.0 / K;
+  const double g0sq = tot * (1.0 / ((double)K * K));
+  if (!(c > 0.0) || !(g0sq > 0.0)) {
+    if (act) beta_out[lane] = 1.0 / K;
+    return true;
+  }
+  if (!__all_sync(0xffffffffu, !act || bd > 0.0)) return false;  // 0 may lie in the hull
+  const double rho = c * sqrt_nr(g0sq);
+  const float rhof = (float)rho, bf = (float)bd;
+  const float Fv = act ? bf + rhof * sqrtf(fmaxf(Gf[lane * K + lane], 0.0f)) : INFINITY;
+  const int k0 = warp_argmin_f(Fv, lane);
+  bool in = lane == k0;
+  float w = in ? 1.0f : 0.0f;
+  float row[kCols];
+  for (int major = 0; major < 4 * K + 4; ++major) {
+    float v = 0.0f;
+    for (int j = 0; j < K; ++j) {
+      const float wj = __shfl_sync(0xffffffffu, w, j);
+      if (act) v = fmaf(Gf[lane * K + j], wj, v);
+    }
+    const float q = warp_sum_f(act ? w * v : 0.0f);
+    if (!(q > 1e-20f)) return false;
+    const float gk = act ? bf + rhof * v / sqrtf(q) : INFINITY;
+    const float lam = warp_sum_f(act ? w * gk : 0.0f);
+    const int jn = warp_argmin_f(gk, lane);
+    if (__shfl_sync(0xffffffffu, gk, jn) >= lam - 1e-6f) break;
+    if (__shfl_sync(0xffffffffu, in ? 1 : 0, jn)) break;
+    if (lane == jn) {
+      in = true;
+      w = 0.0f;
+    }
+    bool settled = false;
+    for (int minor = 0; minor <= K + 1 && !settled; ++minor) {
+      const unsigned smask = __ballot_sync(0xffffffffu, in && act);
+      const int s = __popc(smask);
+      if (s == 0) return false;
+      const int pi = lane < s ? nth_set(smask, lane) : 0;
+      cagrad_rows(Gf, K, smask, lane, 0.0f, 1.0f, __shfl_sync(0xffffffffu, bf, pi), row);
+      if (!warp_gauss_jordan(row, s, lane, 1e-6f)) return false;
+      const float mi = lane < s ? row[kUnk] : 0.0f, ni = lane < s ? row[kUnk + 1] : 0.0f;
+      const float bpi = __shfl_sync(0xffffffffu, bf, pi);
+      const float om = warp_sum_f(mi), on = warp_sum_f(ni), nb = warp_sum_f(lane < s ? ni * bpi : 0.0f);
+      const float D = on * on - om * (nb - rhof * rhof);
+      if (!(om > 0.0f) || !(D > 0.0f)) return false;
+      const float sd = sqrtf(D), lamc = (on + sd) / om;
+      const float zi = (lamc * mi - ni) / sd;                  // lane i < s: support entry i
+      const int rank = __popc(smask & ((1u << lane) - 1u));
+      const float zk_all = __shfl_sync(0xffffffffu, zi, in ? rank : 0);
+      const float z = in ? zk_all : 0.0f;
+      if (__all_sync(0xffffffffu, !in || z > 1e-7f)) {
+        const float zs = warp_sum_f(z);
+        w = z / zs;
+        settled = true;
+        break;
+      }
+      const float t = (in && z <= 1e-7f) ? ((w - z) > 0.0f ? w / (w - z) : 0.0f) : INFINITY;
+      const int drop = warp_argmin_f(t, lane);
+      const float theta = __shfl_sync(0xffffffffu, t, drop);
+      w = in ? (1.0f - theta) * w + theta * z : 0.0f;
+      if (lane == drop || w <= 1e-7f) {
+        in = false;
+        w = 0.0f;
+      }
+    }
+    if (!settled) return false;
+  }
+  // fp64: m = G_SS^-1 1 and n = G_SS^-1 b_S with one refinement step
+  const unsigned smask = __ballot_sync(0xffffffffu, in && act);
+  const int s = __popc(smask);
+  if (s == 0) return false;
+  const int pi = lane < s ? nth_set(smask, lane) : 0;
+  const double bpi = __shfl_sync(0xffffffffu, bd, pi);
+  cagrad_rows(Gf, K, smask, lane, 0.0f, 1.0f, (float)bpi, row);
+  if (!warp_gauss_jordan(row, s, lane, 1e-6f)) return false;
+  double md = lane < s ? (double)row[kUnk] : 0.0, nd = lane < s ? (double)row[kUnk + 1] : 0.0;
+  double rm = 0.0, rn = 0.0;
+  {
+    double am = 0.0, an = 0.0;
+    for (int j = 0; j < s; ++j) {
+      const double mj = __shfl_sync(0xffffffffu, md, j), nj = __shfl_sync(0xffffffffu, nd, j);
+      if (lane < s) {
+        const double a = G[pi * K + nth_set(smask, j)];
+        am = fma(a, mj, am);
+        an = fma(a, nj, an);
+      }
+    }
+    rm = lane < s ? 1.0 - am : 0.0;
+    rn = lane < s ? bpi - an : 0.0;
+  }
+  cagrad_rows(Gf, K, smask, lane, 0.0f, (float)rm, (float)rn, row);
+  if (!warp_gauss_jordan(row, s, lane, 1e-6f)) return false;
+  if (lane < s) {
+    md += (double)row[kUnk];
+    nd += (double)row[kUnk + 1];
+  }
+  double om = md, on = nd, nb = lane < s ? nd * bpi : 0.0;
+  for (int off = 16; off > 0; off >>= 1) {
+    om += __shfl_xor_sync(0xffffffffu, om, off);
+    on += __shfl_xor_sync(0xffffffffu, on, off);
+    nb += __shfl_xor_sync(0xffffffffu, nb, off);
+  }
+  const double D = on * on - om * (nb - rho * rho);
+  if (!(om > 0.0) || !(D > 0.0)) return false;
+  const double sd = sqrt_nr(D), lamc = div_nr(on + sd, om), isd = div_nr(1.0, sd);
+  const double zi = lane < s ? (lamc * md - nd) * isd : 0.0;
+  const int rank = __popc(smask & ((1u << lane) - 1u));
+  const bool ink = act && ((smask >> lane) & 1u);
+  const double zk = __shfl_sync(0xffffffffu, zi, ink ? rank : 0);
+  double wd = (ink && zk > 0.0) ? zk : 0.0;
+  double sum = wd;
+  for (int off = 16; off > 0; off >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, off);
+  wd *= (2.0 - sum);
+  // optimality of the dual (fp32 with a margin, fp64 if marginal), and
+  // beta = 1/K + rho w / ||g_w|| with ||g_w|| in fp64
+  double vd = 0.0;
+  for (int j = 0; j < K; ++j) {
+    const double wj = __shfl_sync(0xffffffffu, wd, j);
+    if (act) vd = fma(G[lane * K + j], wj, vd);
+  }
+  double qd = act ? wd * vd : 0.0;
+  for (int off = 16; off > 0; off >>= 1) qd += __shfl_xor_sync(0xffffffffu, qd, off);
+  if (!(qd > 1e-24)) return false;
+  const double f = div_nr(rho, sqrt_nr(qd));
+  const double gk = act ? fma(f, vd, bd) : 1e300;
+  double lam = act ? wd * gk : 0.0;
+  for (int off = 16; off > 0; off >>= 1) lam += __shfl_xor_sync(0xffffffffu, lam, off);
+  if (!__all_sync(0xffffffffu, !act || ink || gk >= lam - 1e-11)) return false;
+  if (act) beta_out[lane] = fma(f, wd, 1.0 / K);
+  return true;
+}
+
 template <int K>
 __device__ bool solve_fast_k(int rule, const double* G, const float* Gf, const SolveParams& p,
                              int64_t b, int lane, double* beta_out) {
@@ -1093,7 +1445,11 @@ __device__ bool solve_fast_k(int rule, const double* G, const float* Gf, const S
     pcgrad_fast<K>(G, p.seed, p.step, b, lane, beta_out);
     return true;
   }
-  if (K > kEnumMaxK || !(p.flags & BKMOO_FLAG_POLISH)) return false;
+  if (!(p.flags & BKMOO_FLAG_POLISH)) return false;
+  if (rule == BKMOO_MGDA && K > kEnumMaxK) return mgda_wolfe_warp(K, G, Gf, lane, beta_out);
+  if (rule == BKMOO_CAGRAD && K > kEnumMaxK)
+    return cagrad_active_warp(K, G, Gf, p.cagrad_c, lane, beta_out);
+  if (K > kEnumMaxK) return false;
   if (rule == BKMOO_MGDA) {
     if (K < 2 || (K == 2 && (p.flags & BKMOO_FLAG_CLOSED_FORM_K2))) return false;
     return mgda_fast<(K <= kEnumMaxK ? K : 2)>(G, Gf, lane, beta_out);

@@ -79,6 +79,8 @@ def load():
         lib.bkmoo_workspace_init.argtypes = [i32, i32, vp, i64, vp, sz, vp]
         lib.bkmoo_gram.restype = ctypes.c_int
         lib.bkmoo_gram.argtypes = [vp, i32, i32, vp, i64, vp, vp, sz, vp]
+        lib.bkmoo_conflicts.restype = ctypes.c_int
+        lib.bkmoo_conflicts.argtypes = [vp, i32, i64, vp, vp, vp, vp]
         lib.bkmoo_gram_noalloc.restype = ctypes.c_int
         lib.bkmoo_gram_noalloc.argtypes = [vp, i32, i32, vp, i64, vp, vp]
         lib.bkmoo_resolve.restype = ctypes.c_int
@@ -169,6 +171,16 @@ def bkmoo_gram(grads, offsets, out_gram, ws, stream=None):
                              len(off) - 1, out_gram.data_ptr(), ws.data_ptr(),
                              ws.numel() * ws.element_size(),
                              _stream_handle(stream, grads[0].device)), "bkmoo_gram")
+
+
+def bkmoo_conflicts(gram, out_cos=None, out_stats=None, out_conflict=None, stream=None):
+    """Figure 1's conflict statistics from Gram matrices [B, K, K] (fp64, CUDA)."""
+    B, K = int(gram.shape[0]), int(gram.shape[1])
+    _check(load().bkmoo_conflicts(gram.data_ptr(), K, B,
+                                  out_cos.data_ptr() if out_cos is not None else None,
+                                  out_stats.data_ptr() if out_stats is not None else None,
+                                  out_conflict.data_ptr() if out_conflict is not None else None,
+                                  _stream_handle(stream, gram.device)), "bkmoo_conflicts")
 
 
 def bkmoo_gram_noalloc(grads, offsets, out_gram, stream=None):

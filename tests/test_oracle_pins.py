@@ -621,3 +621,34 @@ def test_mgda_frank_wolfe_step_is_exact_line_search():
         j = int(np.argmin(vals))
         assert _obj(G, a1) <= vals[j] + 1e-12 * G.max()
         assert np.abs(a1 - path[j]).max() <= 2e-5
+
+
+# ----------------------------------------------------------------------------
+# Conflict statistics (Figure 1; Eq. 2, Definition A.4)
+# ----------------------------------------------------------------------------
+
+def test_conflicts_closed_forms():
+    e1, e2 = np.array([1.0, 0, 0]), np.array([0, 1.0, 0])
+    cos, st, flag = orc.conflicts(_gram_np([e1, e2]))          # orthogonal
+    np.testing.assert_allclose(cos, np.eye(2), atol=1e-15)
+    assert flag == 0 and st[0] == 0 and st[1] == 0 and st[2] == 0
+    cos, st, flag = orc.conflicts(_gram_np([e1, -2 * e1]))     # opposed
+    assert abs(cos[0, 1] + 1) < 1e-15 and flag == 1 and abs(st[2] + 1) < 1e-15
+    cos, st, flag = orc.conflicts(_gram_np([e1, 3 * e1, e2]))  # 1, 0, 0
+    np.testing.assert_allclose(st, [1 / 3, np.sqrt(2) / 3, 0.0], atol=1e-15)
+    assert flag == 0
+    cos, st, flag = orc.conflicts(_gram_np([e1, np.zeros(3), -e1]))   # zero gradient
+    assert cos[1, 1] == 0 and cos[0, 1] == 0 and flag == 1
+
+
+def test_conflicts_match_materialised_cosines():
+    rng = np.random.default_rng(40)
+    for K in (2, 3, 4, 8, 16):
+        vs = _rand_vectors(rng, K, 50, corr=rng.uniform(-0.9, 0.9), flip_odd=True)
+        cos, st, flag = orc.conflicts(_gram_np(vs))
+        X = np.stack(vs)
+        C = (X @ X.T) / np.outer(np.linalg.norm(X, axis=1), np.linalg.norm(X, axis=1))
+        np.testing.assert_allclose(cos, C, atol=1e-12)
+        pairs = C[np.triu_indices(K, 1)]
+        np.testing.assert_allclose(st, [pairs.mean(), pairs.std(), pairs.min()], atol=1e-12)
+        assert flag == int((pairs < 0).any())

@@ -337,3 +337,33 @@ def test_fused_workspace_mismatch_is_detected():
     assert bool((out == 7.0).all())
     res.resolve(grads, "mgda", out, params=_fused_params())
     assert res.status() == 0
+
+
+@pytest.mark.parametrize("K", [2, 4, 8, 16])
+def test_conflict_statistics(K):
+    """Figure 1 statistics from the GPU Gram against the oracle's (cosines to
+    the Gram tolerance; the conflict flag exactly, except where the most
+    negative cosine is within that tolerance of 0)."""
+    w = _workload(K, "bf16", RAGGED, 120000, seed=90 + K, rho=(-0.6, 0.9), flip=0.3)
+    off = bk.bkmoo_plan(w.param_sizes, w.elem_bytes, w.bucket_bytes)
+    grads = inputs.generate(w, off, DEV)
+    hv = [inputs.host_view(g) for g in grads]
+    B = len(off) - 1
+    res = bk.Resolver(K, torch.bfloat16, off, DEV)
+    G = torch.empty(B, K, K, dtype=torch.float64, device=DEV)
+    res.gram(grads, G)
+    cos = torch.empty(B, K, K, dtype=torch.float32, device=DEV)
+    stats = torch.empty(B, 3, dtype=torch.float32, device=DEV)
+    flag = torch.empty(B, dtype=torch.int32, device=DEV)
+    bk.bkmoo_conflicts(G, cos, stats, flag)
+    torch.cuda.synchronize()
+    cos, stats, flag = cos.cpu().numpy(), stats.cpu().numpy(), flag.cpu().numpy()
+    seen = 0
+    for b in range(B):
+        c_or, s_or, f_or = orc.conflicts(orc.gram(hv, int(off[b]), int(off[b + 1] - off[b])))
+        np.testing.assert_allclose(cos[b], c_or, atol=2e-5)
+        np.testing.assert_allclose(stats[b], s_or, atol=2e-5)
+        if abs(s_or[2]) > 2e-5:
+            assert flag[b] == f_or, b
+        seen += f_or
+    assert seen > 0          # the workload has conflicting buckets
