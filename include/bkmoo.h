@@ -75,7 +75,9 @@ typedef enum { BKMOO_F32 = 0, BKMOO_BF16 = 1 } bkmoo_dtype;
                                           CAGrad)                            */
 #define BKMOO_FLAG_FUSED 0x4u          /* one persistent launch that resolves
                                           bucket after bucket while the
-                                          bucket is still in L2              */
+                                          bucket is still in L2 (K <= 8; for
+                                          larger K the flag is ignored and
+                                          the three-pass path runs)          */
 
 typedef struct {
   int32_t max_iter; /* Frank-Wolfe iterations per bucket (MGDA, CAGrad)     */

@@ -12,6 +12,10 @@
 namespace bkmoo {
 
 constexpr int kMaxK = 16;
+// Largest K the fused persistent kernel is built for: above it the per-thread
+// streaming state (K(K+1)/2 accumulators, K vectors in flight) no longer fits
+// the register file, and the three-pass path runs instead.
+constexpr int kFusedMaxK = 8;
 constexpr int kThreads = 256;              // CTA size of the streaming kernels
 constexpr int kWarps = kThreads / 32;
 constexpr int kVecPerThread = 16;          // 16-byte vectors per thread per Gram chunk
@@ -208,10 +212,10 @@ const void* combine_fn_f32(int K, int dtype_out);
 const void* combine_fn_bf16(int K, int dtype_out);
 
 // Fused kernels, signature (GradPtrs, FusedView, SolveParams, void* out); fused_*.cu.
-const void* fused_fn_f32_k1_8(int K, int dtype_out);
-const void* fused_fn_f32_k9_16(int K, int dtype_out);
-const void* fused_fn_bf16_k1_8(int K, int dtype_out);
-const void* fused_fn_bf16_k9_16(int K, int dtype_out);
+const void* fused_fn_f32_k1_4(int K, int dtype_out);
+const void* fused_fn_f32_k5_8(int K, int dtype_out);
+const void* fused_fn_bf16_k1_4(int K, int dtype_out);
+const void* fused_fn_bf16_k5_8(int K, int dtype_out);
 
 // solve.cu
 cudaError_t launch_solve(const PlanView& v, const SolveParams& p, float* out_weights,

@@ -178,7 +178,7 @@ __device__ __noinline__ void fused_solver_cta(const FusedView& f, const SolvePar
     }
     __syncthreads();
     if (warp == 0) {
-      const int st = solver::solve_bucket_warp(K, G, Gf, prm, b, beta_sh, lane);
+      const int st = solver::solve_bucket_warp<K>(K, G, Gf, prm, b, beta_sh, lane);
       if (lane < K) {
         const float fb = (float)beta_sh[lane];
         v.beta[b * K + lane] = fb;
@@ -453,11 +453,9 @@ __global__ void __launch_bounds__(kThreads, FusedMinBlocks<K>::value)
    (const void*)fused_resolve_kernel<K, DTI, BKMOO_BF16>}
 
 // Eight values of K per translation unit (compiled in parallel).
-#define BKMOO_FUSED_TABLE8(DTI, K0)                                                        \
-  static const void* const kFusedTable[8][2] = {                                           \
+#define BKMOO_FUSED_TABLE4(DTI, K0)                                                        \
+  static const void* const kFusedTable[4][2] = {                                           \
       BKMOO_FUSED_ROW(K0 + 0, DTI), BKMOO_FUSED_ROW(K0 + 1, DTI),                          \
-      BKMOO_FUSED_ROW(K0 + 2, DTI), BKMOO_FUSED_ROW(K0 + 3, DTI),                          \
-      BKMOO_FUSED_ROW(K0 + 4, DTI), BKMOO_FUSED_ROW(K0 + 5, DTI),                          \
-      BKMOO_FUSED_ROW(K0 + 6, DTI), BKMOO_FUSED_ROW(K0 + 7, DTI)}
+      BKMOO_FUSED_ROW(K0 + 2, DTI), BKMOO_FUSED_ROW(K0 + 3, DTI)}
 
 }  // namespace bkmoo

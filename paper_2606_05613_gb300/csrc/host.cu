@@ -91,8 +91,8 @@ const void* combine_fn(int K, int dti, int dto) {
   return dti == BKMOO_F32 ? combine_fn_f32(K, dto) : combine_fn_bf16(K, dto);
 }
 const void* fused_fn(int K, int dti, int dto) {
-  if (dti == BKMOO_F32) return K <= 8 ? fused_fn_f32_k1_8(K, dto) : fused_fn_f32_k9_16(K, dto);
-  return K <= 8 ? fused_fn_bf16_k1_8(K, dto) : fused_fn_bf16_k9_16(K, dto);
+  if (dti == BKMOO_F32) return K <= 4 ? fused_fn_f32_k1_4(K, dto) : fused_fn_f32_k5_8(K, dto);
+  return K <= 4 ? fused_fn_bf16_k1_4(K, dto) : fused_fn_bf16_k5_8(K, dto);
 }
 
 // The fused path: one cooperative (co-resident) launch; the last CTA solves.
@@ -330,7 +330,7 @@ int bkmoo_resolve(const void* const* grads, int32_t K, int32_t in_dtype, const i
   sp.step = prm.step;
   sp.flags = prm.flags;
   if (ev && cudaEventRecord(ev[0], s) != cudaSuccess) return BKMOO_ERR_CUDA;
-  if (prm.flags & BKMOO_FLAG_FUSED) {
+  if ((prm.flags & BKMOO_FLAG_FUSED) && K <= kFusedMaxK) {
     int64_t nmax = 0;
     for (int64_t b = 0; b < n_buckets; ++b)
       if (offsets[b + 1] - offsets[b] > nmax) nmax = offsets[b + 1] - offsets[b];

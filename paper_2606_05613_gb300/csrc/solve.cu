@@ -26,7 +26,7 @@ __global__ void __launch_bounds__(32 * kSolveWarpsPerBlock)
   double* G = Gs[wi];
   double* beta = Bs[wi];
   reduce_bucket(v, b, G, lane);
-  const int st = solve_bucket_warp(K, G, Fs[wi], p, b, beta, lane);
+  const int st = solve_bucket_warp<0>(K, G, Fs[wi], p, b, beta, lane);
   for (int k = lane; k < K; k += 32) {
     const float f = (float)beta[k];
     v.beta[b * K + k] = f;

@@ -1438,7 +1438,19 @@ __device__ bool cagrad_active_warp(int K, const double* G, const float* Gf, doub
   return true;
 }
 
-template <int K>
+// Large-K (K > kEnumMaxK) MGDA and CAGrad: one copy of the lane-parallel
+// active-set solvers per kernel, whatever the number of K cases around it.
+__device__ bool solve_large(int K, int rule, const double* G, const float* Gf,
+                            const SolveParams& p, int lane, double* beta_out) {
+  if (!(p.flags & BKMOO_FLAG_POLISH)) return false;
+  if (rule == BKMOO_MGDA) return mgda_wolfe_warp(K, G, Gf, lane, beta_out);
+  if (rule == BKMOO_CAGRAD) return cagrad_active_warp(K, G, Gf, p.cagrad_c, lane, beta_out);
+  return false;
+}
+
+// kLarge: whether this instantiation carries the large-K solvers itself
+// (the runtime-K dispatch below calls solve_large once, outside its switch).
+template <int K, bool kLarge>
 __device__ bool solve_fast_k(int rule, const double* G, const float* Gf, const SolveParams& p,
                              int64_t b, int lane, double* beta_out) {
   if (rule == BKMOO_PCGRAD) {
@@ -1446,10 +1458,7 @@ __device__ bool solve_fast_k(int rule, const double* G, const float* Gf, const S
     return true;
   }
   if (!(p.flags & BKMOO_FLAG_POLISH)) return false;
-  if (rule == BKMOO_MGDA && K > kEnumMaxK) return mgda_wolfe_warp(K, G, Gf, lane, beta_out);
-  if (rule == BKMOO_CAGRAD && K > kEnumMaxK)
-    return cagrad_active_warp(K, G, Gf, p.cagrad_c, lane, beta_out);
-  if (K > kEnumMaxK) return false;
+  if (K > kEnumMaxK) return kLarge ? solve_large(K, rule, G, Gf, p, lane, beta_out) : false;
   if (rule == BKMOO_MGDA) {
     if (K < 2 || (K == 2 && (p.flags & BKMOO_FLAG_CLOSED_FORM_K2))) return false;
     return mgda_fast<(K <= kEnumMaxK ? K : 2)>(G, Gf, lane, beta_out);
@@ -1463,9 +1472,10 @@ __device__ bool solve_fast_k(int rule, const double* G, const float* Gf, const S
 // after the caller's __syncwarp).
 __device__ bool solve_fast(int K, int rule, const double* G, const float* Gf,
                            const SolveParams& p, int64_t b, int lane, double* beta_out) {
+  if (K > kEnumMaxK && rule != BKMOO_PCGRAD) return solve_large(K, rule, G, Gf, p, lane, beta_out);
   switch (K) {
 #define BKMOO_FAST_CASE(k) \
-  case k: return solve_fast_k<k>(rule, G, Gf, p, b, lane, beta_out);
+  case k: return solve_fast_k<k, false>(rule, G, Gf, p, b, lane, beta_out);
     BKMOO_FAST_CASE(1) BKMOO_FAST_CASE(2) BKMOO_FAST_CASE(3) BKMOO_FAST_CASE(4)
     BKMOO_FAST_CASE(5) BKMOO_FAST_CASE(6) BKMOO_FAST_CASE(7) BKMOO_FAST_CASE(8)
     BKMOO_FAST_CASE(9) BKMOO_FAST_CASE(10) BKMOO_FAST_CASE(11) BKMOO_FAST_CASE(12)
@@ -1482,6 +1492,9 @@ __device__ bool solve_fast(int K, int rule, const double* G, const float* Gf,
 // The whole warp enters with G (K x K) in shared memory; G is normalised in
 // place.  beta_out (shared, K entries) and the returned status are valid on
 // every lane after the call.
+// KC > 0: K is the compile-time constant KC (one solver instantiation);
+// KC = 0: K is a runtime value dispatched over 1..kMaxK.
+template <int KC>
 __device__ int solve_bucket_warp(int K, double* G, float* Gf, const SolveParams& p, int64_t b,
                                  double* beta_out, int lane) {
   // finiteness and the largest diagonal entry from the bit patterns
@@ -1523,7 +1536,11 @@ __device__ int solve_bucket_warp(int K, double* G, float* Gf, const SolveParams&
   SolveParams q = p;
   q.tol = p.tol * top;  // the stopping test is relative to max_k G_kk
   int st = BKMOO_OK;
-  const bool fast = solve_fast(K, q.rule, G, Gf, q, b, lane, beta_out);
+  bool fast;
+  if constexpr (KC > 0)
+    fast = solve_fast_k<KC, true>(q.rule, G, Gf, q, b, lane, beta_out);
+  else
+    fast = solve_fast(K, q.rule, G, Gf, q, b, lane, beta_out);
   if (!fast && lane == 0) {
     double beta[kMaxK];
     switch (q.rule) {
