@@ -162,6 +162,22 @@ class ClockSampler:
                 "reasons": reasons, "samples": len(rows)}
 
 
+def reduce_over_ranks(ms_step, grad_bytes, device):
+    """Whole-job throughput: the gradient bytes of all ranks over the slowest
+    rank's time per step.  Returns (max ms per step, GB/s).  One rank: no
+    collective."""
+    import torch
+    import torch.distributed as dist
+    if not (dist.is_available() and dist.is_initialized()) or dist.get_world_size() == 1:
+        return ms_step, grad_bytes / (ms_step * 1e-3) / GB
+    t = torch.tensor([ms_step], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    u = torch.tensor([float(grad_bytes)], dtype=torch.float64, device=device)
+    dist.all_reduce(u, op=dist.ReduceOp.SUM)
+    ms = float(t.item())
+    return ms, float(u.item()) / (ms * 1e-3) / GB
+
+
 def cpu_baseline(w, offsets, seconds, n_threads=0):
     """The oracle, as it stands, on a bounded sample of the workload's
     buckets (host-generated with the same generator), repeated until about
@@ -345,13 +361,8 @@ def main():
     total_ms = evs[0][0].elapsed_time(evs[-1][3])
     per = np.array([[e4[0].elapsed_time(e4[1]), e4[1].elapsed_time(e4[2]),
                      e4[2].elapsed_time(e4[3])] for e4 in evs])
-    ms_step = total_ms / a.steps
-    if world > 1:
-        t = torch.tensor([ms_step], device=dev)
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        ms_step = float(t.item())
     grad_bytes = w.K * N * w.elem_bytes
-    value = world * grad_bytes / (ms_step * 1e-3) / GB
+    ms_step, value = reduce_over_ranks(total_ms / a.steps, grad_bytes, dev)
 
     peak, peak_kind = _peaks()
     e_in = w.elem_bytes
@@ -416,9 +427,13 @@ def main():
 
 
 def e2e_measure(a, w, off, grads, res, params, dev, tdt):
-    """Host (pinned) gradients -> device -> resolve -> host direction, all
-    inside the timed region, through the Python binding of the C ABI."""
+    """End to end through the public host-memory entry point
+    (bkmoo_resolve_host): page-locked host gradients in, page-locked host
+    direction out, every byte crossing the host link inside the timed region
+    (the call overlaps the copies with the resolve)."""
     import torch
+
+    from paper_2606_05613_gb300 import native as bk
     N = int(off[-1])
     try:
         host = [torch.empty(N, dtype=tdt, pin_memory=True) for _ in range(w.K)]
@@ -428,18 +443,23 @@ def e2e_measure(a, w, off, grads, res, params, dev, tdt):
                 % str(e)[:120]}
     for k in range(w.K):
         host[k].copy_(grads[k])
+    torch.cuda.synchronize(dev)
+    out_dt = bk.BKMOO_F32 if tdt == torch.float32 else bk.BKMOO_BF16
+    # windows of about an eighth of the model, at most 64 Mi elements per
+    # language, never shorter than the longest bucket
+    longest = int((off[1:] - off[:-1]).max())
+    window = max(longest, min(1 << 26, N // 8))
+    staging = torch.empty(res.staging_size(out_dt, window), dtype=torch.uint8, device=dev)
     stream = torch.cuda.current_stream(dev)
-    out = torch.empty(N, dtype=tdt, device=dev)
     params.events = None
 
     def one():
-        for k in range(w.K):
-            grads[k].copy_(host[k], non_blocking=True)
-        res.resolve(grads, a.rule, out, params=params)
-        host_out.copy_(out, non_blocking=True)
+        res.resolve_host(host, a.rule, host_out, staging, params=params)
         stream.synchronize()
 
     one()
+    if res.status() != 0:
+        raise SystemExit("host resolve failed: " + bk.bkmoo_status_string(res.status()))
     t0 = time.perf_counter()
     for _ in range(a.e2e_steps):
         one()
@@ -447,7 +467,9 @@ def e2e_measure(a, w, off, grads, res, params, dev, tdt):
     gb = w.K * N * w.elem_bytes
     return {"value": gb / dt / GB, "unit": "GB/s", "ms_per_step": dt * 1e3,
             "h2d_bytes_per_step": gb, "d2h_bytes_per_step": N * host_out.element_size(),
-            "steps": a.e2e_steps}
+            "steps": a.e2e_steps, "api": "bkmoo_resolve_host",
+            "window_elems": window, "staging_bytes": staging.numel(),
+            "link_GBps": (gb + N * host_out.element_size()) / dt / GB}
 
 
 if __name__ == "__main__":

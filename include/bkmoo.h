@@ -248,6 +248,54 @@ int bkmoo_resolve(const void* const* grads, int32_t K, int32_t in_dtype,
                   size_t ws_bytes, void* stream);
 
 /*
+ * bkmoo_host_staging_size -- device staging bytes bkmoo_resolve_host needs
+ * so that every window holds at least max(window_elems, the largest bucket)
+ * elements per language.  Host only, pure.  Writes *bytes.
+ */
+int bkmoo_host_staging_size(int32_t K, int32_t in_dtype, int32_t out_dtype,
+                            const int64_t* offsets, int64_t n_buckets, int64_t window_elems,
+                            size_t* bytes);
+
+/*
+ * bkmoo_resolve_host -- bkmoo_resolve for gradients held in HOST memory, the
+ * direction written back to host memory.  It follows the per-bucket loop of
+ * Algorithm 1 -- bring a bucket's K gradients to the device, resolve it,
+ * send its direction on and free the bucket's device copy -- so that device
+ * memory holds only a bounded window of buckets, not the K full gradients.
+ *
+ * Buckets go through two device staging slots in windows of whole buckets:
+ * while window w is resolved (Gram -> rule -> combination on `stream`, the
+ * same kernels and the same per-chunk arithmetic as bkmoo_resolve, so beta
+ * and the direction are bit-identical to it), window w+1 is copied in and
+ * window w-1's direction copied out on two internal copy streams, created
+ * and destroyed by the call.  Work already queued on `stream` comes first;
+ * `stream` completes only after the last byte reaches host_out.
+ *
+ * host_grads: host array of K host pointers (16-byte aligned), N elements
+ *   each.  Page-locked memory (cudaHostAlloc / cudaHostRegister) lets the
+ *   copies overlap; pageable memory gives the same results more slowly.
+ * host_out: host, N elements of out_dtype; may be exactly one of host_grads
+ *   (same dtype); any other overlap is BKMOO_ERR_INVALID.
+ * out_weights, out_status, ws, ws_bytes, rule, p: as in bkmoo_resolve (device
+ *   buffers; ws initialised for this plan).  p->events and
+ *   BKMOO_FLAG_FUSED are ignored.
+ * staging: device, 256-byte aligned, staging_bytes long.  It holds two
+ *   slots of K input regions and one output region of
+ *   round_up(cap e + 16, 256) bytes each (e the region's element size); cap,
+ *   the window length in elements per language, is the largest that fits.
+ *   A bucket longer than cap is BKMOO_ERR_WORKSPACE (bkmoo_host_staging_size
+ *   gives the size for a chosen cap).  Larger staging means fewer, longer
+ *   windows.  Calls that share a staging buffer or a workspace must not
+ *   overlap on the GPU.
+ * Returns BKMOO_OK once everything is queued.
+ */
+int bkmoo_resolve_host(const void* const* host_grads, int32_t K, int32_t in_dtype,
+                       const int64_t* offsets, int64_t n_buckets, int32_t rule,
+                       const bkmoo_params* p, void* host_out, int32_t out_dtype,
+                       float* out_weights, int32_t* out_status, void* ws, size_t ws_bytes,
+                       void* staging, size_t staging_bytes, void* stream);
+
+/*
  * bkmoo_workspace_status -- synchronise `stream` and read the workspace
  * status word: BKMOO_OK, or the first device-side error recorded since the
  * last bkmoo_gram / bkmoo_resolve started (BKMOO_ERR_WORKSPACE,

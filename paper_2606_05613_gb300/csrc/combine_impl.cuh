@@ -62,8 +62,8 @@ __global__ void __launch_bounds__(kThreads) combine_kernel(const GradPtrs g, con
   constexpr int IB = 16 / EPV;  // input bytes per element
   if (!header_ok(v)) return;    // the Gram pass already recorded the error
 
-  int64_t b = 0;
-  for (int64_t w = blockIdx.x; w < v.n_chunks; w += gridDim.x) {
+  int64_t b = v.b_lo;
+  for (int64_t w = v.c_lo + blockIdx.x; w < v.c_hi; w += gridDim.x) {
     b = find_bucket(v.chunk_prefix, v.n_buckets, w, b);
     float beta[K];
 #pragma unroll

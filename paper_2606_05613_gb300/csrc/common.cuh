@@ -99,7 +99,19 @@ struct PlanView {
   uint64_t plan_hash;
   int32_t K;
   int32_t in_dtype;
+  // The part of the plan one launch works on: chunks [c_lo, c_hi) of buckets
+  // [b_lo, b_hi) (the whole plan except in the windowed host-memory path).
+  int64_t c_lo, c_hi;
+  int64_t b_lo, b_hi;
 };
+
+// Whole-plan window of a view whose n_buckets and n_chunks are set.
+__host__ __device__ inline void full_window(PlanView& v) {
+  v.c_lo = 0;
+  v.c_hi = v.n_chunks;
+  v.b_lo = 0;
+  v.b_hi = v.n_buckets;
+}
 
 // The fused path's view: the plan plus the synchronisation arrays.
 struct FusedView {

@@ -97,8 +97,8 @@ __global__ void __launch_bounds__(kThreads) gram_partials_kernel(const GradPtrs 
     if (blockIdx.x == 0 && threadIdx.x == 0) record_error(v.hdr, BKMOO_ERR_WORKSPACE);
     return;
   }
-  int64_t b = 0;
-  for (int64_t w = blockIdx.x; w < v.n_chunks; w += gridDim.x) {
+  int64_t b = v.b_lo;
+  for (int64_t w = v.c_lo + blockIdx.x; w < v.c_hi; w += gridDim.x) {
     b = find_bucket(v.chunk_prefix, v.n_buckets, w, b);
     const int64_t be = v.offsets[b + 1];
     const int64_t s = v.offsets[b] + (w - v.chunk_prefix[b]) * v.chunk_elems;

@@ -165,25 +165,94 @@ int prepare(const void* const* grads, int32_t K, int32_t dt, const int64_t* offs
   v->plan_hash = plan_hash(K, dt, offsets, B);
   v->K = K;
   v->in_dtype = dt;
+  full_window(*v);
   std::memset(g, 0, sizeof(*g));
   for (int k = 0; k < K; ++k) g->p[k] = grads[k];
   return BKMOO_OK;
 }
 
-int launch_gram_pass(const GradPtrs& g, const PlanView& v, cudaStream_t s) {
-  if (cudaMemsetAsync(&v.hdr->status, 0, sizeof(int32_t), s) != cudaSuccess)
+// Gram pass over the view's window; `reset` clears the workspace status word
+// first (once per call of the C ABI, not per window).
+int launch_gram_pass(const GradPtrs& g, const PlanView& v, cudaStream_t s, bool reset = true) {
+  if (reset && cudaMemsetAsync(&v.hdr->status, 0, sizeof(int32_t), s) != cudaSuccess)
     return BKMOO_ERR_CUDA;
-  if (v.n_chunks == 0) return BKMOO_OK;
+  const int64_t nch = v.c_hi - v.c_lo;
+  if (nch <= 0) return BKMOO_OK;
   const void* fn = gram_fn(v.K, v.in_dtype);
   int grid = 0;
   if (persistent_grid(fn, kThreads, &grid) != cudaSuccess) return BKMOO_ERR_CUDA;
-  if (grid > v.n_chunks) grid = (int)v.n_chunks;
+  if (grid > nch) grid = (int)nch;
   GradPtrs ga = g;
   PlanView va = v;
   void* args[] = {&ga, &va};
   if (cudaLaunchKernel(fn, dim3(grid), dim3(kThreads), args, 0, s) != cudaSuccess)
     return BKMOO_ERR_CUDA;
   return BKMOO_OK;
+}
+
+int launch_combine(const GradPtrs& g, const PlanView& v, void* out, int32_t out_dtype,
+                   cudaStream_t s) {
+  const int64_t nch = v.c_hi - v.c_lo;
+  if (nch <= 0) return BKMOO_OK;
+  const void* fn = combine_fn(v.K, v.in_dtype, out_dtype);
+  int grid = 0;
+  if (persistent_grid(fn, kThreads, &grid) != cudaSuccess) return BKMOO_ERR_CUDA;
+  if (grid > nch) grid = (int)nch;
+  PlanView va = v;
+  GradPtrs ga = g;
+  void* outp = out;
+  void* args[] = {&ga, &va, &outp};
+  if (cudaLaunchKernel(fn, dim3(grid), dim3(kThreads), args, 0, s) != cudaSuccess)
+    return BKMOO_ERR_CUDA;
+  return BKMOO_OK;
+}
+
+bool params_ok(const bkmoo_params& p) {
+  return p.max_iter >= 0 && p.cagrad_c >= 0.0 && p.cagrad_c < 1.0 && p.tol >= 0.0;
+}
+
+SolveParams solve_params(int32_t rule, const bkmoo_params& prm) {
+  SolveParams sp;
+  sp.rule = rule;
+  sp.max_iter = prm.max_iter;
+  sp.tol = prm.tol;
+  sp.cagrad_c = prm.cagrad_c;
+  sp.seed = prm.seed;
+  sp.step = prm.step;
+  sp.flags = prm.flags;
+  return sp;
+}
+
+// ---------------------------------------------------------------------------
+// Host-memory path (bkmoo_resolve_host): windows of whole buckets streamed
+// through two device staging slots.
+// ---------------------------------------------------------------------------
+
+constexpr int kHostSlots = 2;
+
+// Each slot has K input regions and one output region, each 256-byte
+// aligned, with one 16-byte vector of slack so that a window may start at
+// any element and still keep vector alignment.
+size_t region_bytes(int64_t elems, int32_t dt) {
+  return align256((size_t)elems * elem_bytes(dt) + 16);
+}
+
+size_t staging_bytes_for(int32_t K, int32_t dti, int32_t dto, int64_t elems) {
+  return (size_t)kHostSlots * ((size_t)K * region_bytes(elems, dti) + region_bytes(elems, dto));
+}
+
+// Elements of one language a slot holds for a staging buffer of `bytes`: the
+// largest cap with staging_bytes_for(cap) <= bytes.
+int64_t slot_capacity(int32_t K, int32_t dti, int32_t dto, size_t bytes) {
+  const int64_t per_elem = K * elem_bytes(dti) + elem_bytes(dto);
+  int64_t lo = 0, hi = (int64_t)(bytes / kHostSlots) / per_elem + 1;  // fits, does not fit
+  if (staging_bytes_for(K, dti, dto, 0) > bytes) return 0;
+  while (hi - lo > 1) {
+    const int64_t mid = lo + (hi - lo) / 2;
+    if (staging_bytes_for(K, dti, dto, mid) <= bytes) lo = mid;
+    else hi = mid;
+  }
+  return lo;
 }
 
 }  // namespace
@@ -306,8 +375,7 @@ int bkmoo_resolve(const void* const* grads, int32_t K, int32_t in_dtype, const i
   bkmoo_params prm;
   if (p) prm = *p;
   else bkmoo_default_params(&prm);
-  if (prm.max_iter < 0 || !(prm.cagrad_c >= 0.0 && prm.cagrad_c < 1.0) || !(prm.tol >= 0.0))
-    return BKMOO_ERR_INVALID;
+  if (!params_ok(prm)) return BKMOO_ERR_INVALID;
   PlanView v;
   GradPtrs g;
   int r = prepare(grads, K, in_dtype, offsets, n_buckets, ws, ws_bytes, &v, &g);
@@ -321,14 +389,7 @@ int bkmoo_resolve(const void* const* grads, int32_t K, int32_t in_dtype, const i
   }
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   cudaEvent_t* ev = static_cast<cudaEvent_t*>(prm.events);
-  SolveParams sp;
-  sp.rule = rule;
-  sp.max_iter = prm.max_iter;
-  sp.tol = prm.tol;
-  sp.cagrad_c = prm.cagrad_c;
-  sp.seed = prm.seed;
-  sp.step = prm.step;
-  sp.flags = prm.flags;
+  const SolveParams sp = solve_params(rule, prm);
   if (ev && cudaEventRecord(ev[0], s) != cudaSuccess) return BKMOO_ERR_CUDA;
   if ((prm.flags & BKMOO_FLAG_FUSED) && K <= kFusedMaxK) {
     int64_t nmax = 0;
@@ -346,21 +407,149 @@ int bkmoo_resolve(const void* const* grads, int32_t K, int32_t in_dtype, const i
   if (ev && cudaEventRecord(ev[1], s) != cudaSuccess) return BKMOO_ERR_CUDA;
   if (launch_solve(v, sp, out_weights, out_status, s) != cudaSuccess) return BKMOO_ERR_CUDA;
   if (ev && cudaEventRecord(ev[2], s) != cudaSuccess) return BKMOO_ERR_CUDA;
-  if (v.n_chunks == 0) {
-    if (ev && cudaEventRecord(ev[3], s) != cudaSuccess) return BKMOO_ERR_CUDA;
-    return BKMOO_OK;
-  }
-  const void* fn = combine_fn(K, in_dtype, out_dtype);
-  int grid = 0;
-  if (persistent_grid(fn, kThreads, &grid) != cudaSuccess) return BKMOO_ERR_CUDA;
-  if (grid > v.n_chunks) grid = (int)v.n_chunks;
-  PlanView va = v;
-  GradPtrs ga = g;
-  void* outp = out_dir;
-  void* args[] = {&ga, &va, &outp};
-  if (cudaLaunchKernel(fn, dim3(grid), dim3(kThreads), args, 0, s) != cudaSuccess)
-    return BKMOO_ERR_CUDA;
+  r = launch_combine(g, v, out_dir, out_dtype, s);
+  if (r != BKMOO_OK) return r;
   if (ev && cudaEventRecord(ev[3], s) != cudaSuccess) return BKMOO_ERR_CUDA;
+  return BKMOO_OK;
+}
+
+int bkmoo_host_staging_size(int32_t K, int32_t in_dtype, int32_t out_dtype,
+                            const int64_t* offsets, int64_t n_buckets, int64_t window_elems,
+                            size_t* bytes) {
+  if (!bytes || K < 1 || K > kMaxK || !dtype_ok(in_dtype) || !dtype_ok(out_dtype) ||
+      !offsets_ok(offsets, n_buckets) || window_elems < 0)
+    return BKMOO_ERR_INVALID;
+  int64_t w = window_elems;
+  for (int64_t b = 0; b < n_buckets; ++b)
+    if (offsets[b + 1] - offsets[b] > w) w = offsets[b + 1] - offsets[b];
+  *bytes = staging_bytes_for(K, in_dtype, out_dtype, w);
+  return BKMOO_OK;
+}
+
+int bkmoo_resolve_host(const void* const* host_grads, int32_t K, int32_t in_dtype,
+                       const int64_t* offsets, int64_t n_buckets, int32_t rule,
+                       const bkmoo_params* p, void* host_out, int32_t out_dtype,
+                       float* out_weights, int32_t* out_status, void* ws, size_t ws_bytes,
+                       void* staging, size_t staging_bytes, void* stream) {
+  if (rule < BKMOO_MGDA || rule > BKMOO_MEAN || !dtype_ok(out_dtype) || !host_out || !staging ||
+      !aligned(staging, 256))
+    return BKMOO_ERR_INVALID;
+  bkmoo_params prm;
+  if (p) prm = *p;
+  else bkmoo_default_params(&prm);
+  if (!params_ok(prm)) return BKMOO_ERR_INVALID;
+  // The kernels address the staging slots, never the host buffers; `prepare`
+  // checks the plan and workspace (its pointer checks see the host pointers).
+  PlanView v;
+  GradPtrs unused;
+  int r = prepare(host_grads, K, in_dtype, offsets, n_buckets, ws, ws_bytes, &v, &unused);
+  if (r != BKMOO_OK) return r;
+  const int ei = elem_bytes(in_dtype), eo = elem_bytes(out_dtype);
+  const int64_t N = offsets[n_buckets];
+  {  // host_out may be exactly one gradient (same dtype); any other overlap is refused.
+    const uintptr_t o0 = (uintptr_t)host_out, o1 = o0 + (uintptr_t)N * eo;
+    for (int k = 0; k < K; ++k) {
+      const uintptr_t g0 = (uintptr_t)host_grads[k], g1 = g0 + (uintptr_t)N * ei;
+      if (o0 < g1 && g0 < o1 && !(o0 == g0 && out_dtype == in_dtype)) return BKMOO_ERR_INVALID;
+    }
+  }
+  const int64_t cap = slot_capacity(K, in_dtype, out_dtype, staging_bytes);
+  for (int64_t b = 0; b < n_buckets; ++b)
+    if (offsets[b + 1] - offsets[b] > cap) return BKMOO_ERR_WORKSPACE;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if (cudaMemsetAsync(&v.hdr->status, 0, sizeof(int32_t), s) != cudaSuccess)
+    return BKMOO_ERR_CUDA;
+  if (n_buckets == 0) return BKMOO_OK;
+  const SolveParams sp = solve_params(rule, prm);
+
+  // Slot layout: K input regions then the output region, each of
+  // region_bytes(cap) bytes.
+  const size_t rin = region_bytes(cap, in_dtype), rout = region_bytes(cap, out_dtype);
+  const size_t slot_bytes = (size_t)K * rin + rout;
+  char* const stage = static_cast<char*>(staging);
+  const int vec_in = 16 / ei;  // elements per 16-byte input vector
+
+  // Copy streams and events live for this call only; destroying them while
+  // work is queued is legal (their resources go once the work completes).
+  cudaStream_t h2d = nullptr, d2h = nullptr;
+  cudaEvent_t ev_start = nullptr, in_ready[kHostSlots] = {}, in_free[kHostSlots] = {},
+              out_ready[kHostSlots] = {}, out_free[kHostSlots] = {};
+  bool ok = cudaStreamCreateWithFlags(&h2d, cudaStreamNonBlocking) == cudaSuccess &&
+            cudaStreamCreateWithFlags(&d2h, cudaStreamNonBlocking) == cudaSuccess &&
+            cudaEventCreateWithFlags(&ev_start, cudaEventDisableTiming) == cudaSuccess;
+  for (int i = 0; ok && i < kHostSlots; ++i)
+    ok = cudaEventCreateWithFlags(&in_ready[i], cudaEventDisableTiming) == cudaSuccess &&
+         cudaEventCreateWithFlags(&in_free[i], cudaEventDisableTiming) == cudaSuccess &&
+         cudaEventCreateWithFlags(&out_ready[i], cudaEventDisableTiming) == cudaSuccess &&
+         cudaEventCreateWithFlags(&out_free[i], cudaEventDisableTiming) == cudaSuccess;
+  // Both copy streams start after the work already queued on `stream`.
+  ok = ok && cudaEventRecord(ev_start, s) == cudaSuccess &&
+       cudaStreamWaitEvent(h2d, ev_start, 0) == cudaSuccess &&
+       cudaStreamWaitEvent(d2h, ev_start, 0) == cudaSuccess;
+
+  const int64_t ch = v.chunk_elems;
+  int64_t b0 = 0, c_next = 0;
+  for (int64_t win = 0; ok && b0 < n_buckets; ++win) {
+    // the window: whole buckets b0 .. b1-1, at most `cap` elements
+    int64_t b1 = b0 + 1;
+    while (b1 < n_buckets && offsets[b1 + 1] - offsets[b0] <= cap) ++b1;
+    const int slot = (int)(win % kHostSlots);
+    const int64_t lo = offsets[b0], hi = offsets[b1], n = hi - lo;
+    // element `lo` sits at the same offset within a 16-byte vector as in a
+    // 16-byte-aligned buffer, so the kernels' vector/scalar split holds
+    const int64_t base = lo / vec_in * vec_in;
+    char* sin = stage + (size_t)slot * slot_bytes;
+    char* sout = sin + (size_t)K * rin;
+    if (win >= kHostSlots) ok = ok && cudaStreamWaitEvent(h2d, in_free[slot], 0) == cudaSuccess;
+    for (int k = 0; ok && k < K; ++k)
+      ok = cudaMemcpyAsync(sin + (size_t)k * rin + (size_t)(lo - base) * ei,
+                           static_cast<const char*>(host_grads[k]) + (size_t)lo * ei,
+                           (size_t)n * ei, cudaMemcpyHostToDevice, h2d) == cudaSuccess;
+    ok = ok && cudaEventRecord(in_ready[slot], h2d) == cudaSuccess;
+
+    // Kernel pointers are shifted so that global element i of the plan is
+    // addressed at (region + (i - base) * e): only [lo, hi) is touched.
+    GradPtrs gw;
+    std::memset(&gw, 0, sizeof gw);
+    for (int k = 0; k < K; ++k)
+      gw.p[k] = reinterpret_cast<const void*>((uintptr_t)(sin + (size_t)k * rin) -
+                                              (uintptr_t)base * ei);
+    void* outw = reinterpret_cast<void*>((uintptr_t)sout - (uintptr_t)base * eo);
+    PlanView vw = v;
+    vw.b_lo = b0;
+    vw.b_hi = b1;
+    // chunk range of the window: chunks are numbered bucket by bucket
+    vw.c_lo = c_next;
+    for (int64_t b = b0; b < b1; ++b) c_next += (offsets[b + 1] - offsets[b] + ch - 1) / ch;
+    vw.c_hi = c_next;
+    ok = ok && cudaStreamWaitEvent(s, in_ready[slot], 0) == cudaSuccess;
+    if (win >= kHostSlots) ok = ok && cudaStreamWaitEvent(s, out_free[slot], 0) == cudaSuccess;
+    if (ok) r = launch_gram_pass(gw, vw, s, false);
+    ok = ok && r == BKMOO_OK && launch_solve(vw, sp, out_weights, out_status, s) == cudaSuccess;
+    if (ok) r = launch_combine(gw, vw, outw, out_dtype, s);
+    ok = ok && r == BKMOO_OK && cudaEventRecord(in_free[slot], s) == cudaSuccess &&
+         cudaEventRecord(out_ready[slot], s) == cudaSuccess;
+
+    ok = ok && cudaStreamWaitEvent(d2h, out_ready[slot], 0) == cudaSuccess &&
+         cudaMemcpyAsync(static_cast<char*>(host_out) + (size_t)lo * eo,
+                         sout + (size_t)(lo - base) * eo, (size_t)n * eo,
+                         cudaMemcpyDeviceToHost, d2h) == cudaSuccess &&
+         cudaEventRecord(out_free[slot], d2h) == cudaSuccess;
+    b0 = b1;
+  }
+  // `stream` completes only after the last copy back.
+  ok = ok && cudaEventRecord(ev_start, d2h) == cudaSuccess &&
+       cudaStreamWaitEvent(s, ev_start, 0) == cudaSuccess;
+  if (h2d) cudaStreamDestroy(h2d);
+  if (d2h) cudaStreamDestroy(d2h);
+  if (ev_start) cudaEventDestroy(ev_start);
+  for (int i = 0; i < kHostSlots; ++i) {
+    if (in_ready[i]) cudaEventDestroy(in_ready[i]);
+    if (in_free[i]) cudaEventDestroy(in_free[i]);
+    if (out_ready[i]) cudaEventDestroy(out_ready[i]);
+    if (out_free[i]) cudaEventDestroy(out_free[i]);
+  }
+  if (!ok) return r != BKMOO_OK ? r : BKMOO_ERR_CUDA;
   return BKMOO_OK;
 }
 

@@ -162,6 +162,7 @@ extern "C" int bkmoo_gram_noalloc(const void* const* grads, int32_t K, int32_t i
   v.plan_hash = t.hdr.plan_hash;
   v.K = K;
   v.in_dtype = in_dtype;
+  full_window(v);
   GradPtrs g;
   std::memset(&g, 0, sizeof g);
   for (int k = 0; k < K; ++k) g.p[k] = grads[k];

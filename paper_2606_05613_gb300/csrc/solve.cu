@@ -16,8 +16,8 @@ __global__ void __launch_bounds__(32 * kSolveWarpsPerBlock)
   __shared__ double Bs[kSolveWarpsPerBlock][kMaxK];
   __shared__ float Fs[kSolveWarpsPerBlock][kMaxK * kMaxK];
   const int lane = threadIdx.x & 31, wi = threadIdx.x >> 5;
-  const int64_t b = (int64_t)blockIdx.x * kSolveWarpsPerBlock + wi;
-  if (b >= v.n_buckets) return;
+  const int64_t b = v.b_lo + (int64_t)blockIdx.x * kSolveWarpsPerBlock + wi;
+  if (b >= v.b_hi) return;
   const int K = v.K;
   if (!header_ok(v)) {
     if (lane == 0 && out_status) out_status[b] = BKMOO_ERR_WORKSPACE;
@@ -52,8 +52,8 @@ __global__ void __launch_bounds__(32 * kSolveWarpsPerBlock)
 
 cudaError_t launch_solve(const PlanView& v, const SolveParams& p, float* out_weights,
                          int32_t* out_status, cudaStream_t s) {
-  if (v.n_buckets == 0) return cudaSuccess;
-  const int64_t grid = (v.n_buckets + kSolveWarpsPerBlock - 1) / kSolveWarpsPerBlock;
+  if (v.b_hi <= v.b_lo) return cudaSuccess;
+  const int64_t grid = (v.b_hi - v.b_lo + kSolveWarpsPerBlock - 1) / kSolveWarpsPerBlock;
   solve_kernel<<<(unsigned)grid, 32 * kSolveWarpsPerBlock, 0, s>>>(v, p, out_weights, out_status);
   return cudaGetLastError();
 }

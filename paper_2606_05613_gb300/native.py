@@ -86,6 +86,12 @@ def load():
         lib.bkmoo_resolve.restype = ctypes.c_int
         lib.bkmoo_resolve.argtypes = [vp, i32, i32, vp, i64, i32, ctypes.POINTER(bkmoo_params),
                                       vp, i32, vp, vp, vp, sz, vp]
+        lib.bkmoo_host_staging_size.restype = ctypes.c_int
+        lib.bkmoo_host_staging_size.argtypes = [i32, i32, i32, vp, i64, i64, ctypes.POINTER(sz)]
+        lib.bkmoo_resolve_host.restype = ctypes.c_int
+        lib.bkmoo_resolve_host.argtypes = [vp, i32, i32, vp, i64, i32,
+                                           ctypes.POINTER(bkmoo_params), vp, i32, vp, vp, vp, sz,
+                                           vp, sz, vp]
         lib.bkmoo_workspace_status.restype = ctypes.c_int
         lib.bkmoo_workspace_status.argtypes = [vp, vp, ctypes.POINTER(i32)]
         lib.bkmoo_status_string.restype = ctypes.c_char_p
@@ -211,6 +217,40 @@ def bkmoo_resolve(grads, offsets, rule, out_dir, ws, params=None, out_weights=No
                                 _stream_handle(stream, grads[0].device)), "bkmoo_resolve")
 
 
+def bkmoo_host_staging_size(K: int, in_dtype: int, out_dtype: int, offsets,
+                            window_elems: int = 0) -> int:
+    off = _offsets_array(offsets)
+    n = ctypes.c_size_t(0)
+    _check(load().bkmoo_host_staging_size(K, in_dtype, out_dtype, off.ctypes.data, len(off) - 1,
+                                          window_elems, ctypes.byref(n)),
+           "bkmoo_host_staging_size")
+    return int(n.value)
+
+
+def bkmoo_resolve_host(host_grads, offsets, rule, host_out, ws, staging, params=None,
+                       out_weights=None, out_status=None, stream=None):
+    """host_grads / host_out: contiguous CPU tensors (page-locked for overlap);
+    ws, staging, out_weights, out_status: CUDA tensors."""
+    if isinstance(rule, str):
+        rule = RULES[rule]
+    if not host_grads:
+        raise ValueError("need at least one gradient")
+    for g in list(host_grads) + [host_out]:
+        if g.is_cuda or not g.is_contiguous():
+            raise ValueError("host_grads and host_out must be contiguous CPU tensors")
+    off = _offsets_array(offsets)
+    ptrs = (ctypes.c_void_p * len(host_grads))(*[g.data_ptr() for g in host_grads])
+    p = params if params is not None else bkmoo_default_params()
+    _check(load().bkmoo_resolve_host(ptrs, len(host_grads), _dtype_code(host_grads[0]),
+                                     off.ctypes.data, len(off) - 1, rule, ctypes.byref(p),
+                                     host_out.data_ptr(), _dtype_code(host_out),
+                                     out_weights.data_ptr() if out_weights is not None else None,
+                                     out_status.data_ptr() if out_status is not None else None,
+                                     ws.data_ptr(), ws.numel() * ws.element_size(),
+                                     staging.data_ptr(), staging.numel() * staging.element_size(),
+                                     _stream_handle(stream, ws.device)), "bkmoo_resolve_host")
+
+
 def bkmoo_workspace_status(ws, stream=None) -> int:
     st = ctypes.c_int32(0)
     _check(load().bkmoo_workspace_status(ws.data_ptr(), _stream_handle(stream, ws.device),
@@ -249,6 +289,15 @@ class Resolver:
                 stream=None):
         bkmoo_resolve(grads, self.offsets, rule, out_dir, self.ws, params, out_weights,
                       out_status, stream)
+
+    def resolve_host(self, host_grads, rule, host_out, staging, params=None, out_weights=None,
+                     out_status=None, stream=None):
+        bkmoo_resolve_host(host_grads, self.offsets, rule, host_out, self.ws, staging, params,
+                           out_weights, out_status, stream)
+
+    def staging_size(self, out_dtype: int, window_elems: int = 0) -> int:
+        return bkmoo_host_staging_size(self.K, self.in_dtype, out_dtype, self.offsets,
+                                       window_elems)
 
     def gram(self, grads, out_gram, stream=None):
         bkmoo_gram(grads, self.offsets, out_gram, self.ws, stream)

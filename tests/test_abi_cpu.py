@@ -154,3 +154,59 @@ def test_resolve_rejects_bad_arguments_without_launch():
     q = bk.bkmoo_default_params()
     q.max_iter = -1
     assert call(p=ctypes.byref(q)) == bk.BKMOO_ERR_INVALID
+
+
+def test_host_staging_size():
+    """Two slots, each K input regions and one output region of the largest
+    of (window, longest bucket) elements plus 16 bytes, 256-byte aligned."""
+    off = np.array([0, 1000, 2500, 2600], dtype=np.int64)
+
+    def expect(K, ei, eo, n):
+        r = lambda e: (n * e + 16 + 255) // 256 * 256
+        return 2 * (K * r(ei) + r(eo))
+
+    assert bk.bkmoo_host_staging_size(4, bk.BKMOO_BF16, bk.BKMOO_BF16, off) == expect(4, 2, 2, 1500)
+    assert bk.bkmoo_host_staging_size(3, bk.BKMOO_F32, bk.BKMOO_BF16, off, 10**6) == \
+        expect(3, 4, 2, 10**6)
+    with pytest.raises(bk.BkmooError):
+        bk.bkmoo_host_staging_size(0, bk.BKMOO_F32, bk.BKMOO_F32, off)
+    with pytest.raises(bk.BkmooError):
+        bk.bkmoo_host_staging_size(4, bk.BKMOO_F32, 3, off)
+    with pytest.raises(bk.BkmooError):
+        bk.bkmoo_host_staging_size(4, bk.BKMOO_F32, bk.BKMOO_F32, off, -1)
+
+
+def test_resolve_host_rejects_bad_arguments_without_launch():
+    """Argument errors of bkmoo_resolve_host are returned before any CUDA
+    call (fake, aligned addresses)."""
+    lib = bk.load()
+    off = np.array([0, 1000, 2500], dtype=np.int64)
+    base = 1 << 40
+    grads = (ctypes.c_void_p * 4)(*[base + i * (1 << 20) for i in range(4)])
+    ws = ctypes.c_void_p(base + (1 << 30))
+    out = ctypes.c_void_p(base + (1 << 31))
+    stg = ctypes.c_void_p(base + (1 << 32))
+    p = bk.bkmoo_default_params()
+    need = bk.bkmoo_host_staging_size(4, 0, 0, off)
+
+    def call(**kw):
+        a = dict(grads=grads, K=4, dt=0, off=off.ctypes.data, B=2, rule=0, p=ctypes.byref(p),
+                 out=out, odt=0, ws=ws, wsb=1 << 30, stg=stg, stgb=need)
+        a.update(kw)
+        return lib.bkmoo_resolve_host(a["grads"], a["K"], a["dt"], a["off"], a["B"], a["rule"],
+                                      a["p"], a["out"], a["odt"], None, None, a["ws"], a["wsb"],
+                                      a["stg"], a["stgb"], None)
+
+    assert call(K=0) == bk.BKMOO_ERR_INVALID
+    assert call(rule=4) == bk.BKMOO_ERR_INVALID
+    assert call(odt=2) == bk.BKMOO_ERR_INVALID
+    assert call(out=None) == bk.BKMOO_ERR_INVALID
+    assert call(stg=None) == bk.BKMOO_ERR_INVALID
+    assert call(stg=ctypes.c_void_p(base + (1 << 32) + 128)) == bk.BKMOO_ERR_INVALID  # 256-B
+    assert call(wsb=64) == bk.BKMOO_ERR_WORKSPACE
+    assert call(stgb=need - 512) == bk.BKMOO_ERR_WORKSPACE        # a bucket does not fit a slot
+    assert call(out=ctypes.c_void_p(base + 256)) == bk.BKMOO_ERR_INVALID     # partial overlap
+    assert call(out=ctypes.c_void_p(base), odt=1) == bk.BKMOO_ERR_INVALID    # in place, other dtype
+    q = bk.bkmoo_default_params()
+    q.cagrad_c = -0.5
+    assert call(p=ctypes.byref(q)) == bk.BKMOO_ERR_INVALID

@@ -265,6 +265,37 @@ def test_all_zero_bucket_gives_zero_direction():
         assert torch.count_nonzero(out).item() == 0
 
 
+@pytest.mark.parametrize("dt", ["f32", "bf16"])
+def test_global_variant_is_one_bucket(dt):
+    """The conventional (global) MOO is the trivial partition into one bucket
+    (Section 3.1; Table 2 compares the two): its Gram is the sum of the
+    bucket Grams of any finer partition (inner products decompose over
+    disjoint blocks), and its resolve matches the oracle's one-bucket
+    resolve."""
+    K = 4
+    w = _workload(K, dt, RAGGED, 150000, seed=77, flip=0.3)
+    off = bk.bkmoo_plan(w.param_sizes, w.elem_bytes, w.bucket_bytes)
+    assert len(off) > 3
+    grads = inputs.generate(w, off, DEV)
+    hv = [inputs.host_view(g) for g in grads]
+    N = int(off[-1])
+    one = np.array([0, N], dtype=np.int64)
+    Gb = torch.empty(len(off) - 1, K, K, dtype=torch.float64, device=DEV)
+    bk.Resolver(K, _tdt(dt), off, DEV).gram(grads, Gb)
+    res1 = bk.Resolver(K, _tdt(dt), one, DEV)
+    G1 = torch.empty(1, K, K, dtype=torch.float64, device=DEV)
+    res1.gram(grads, G1)
+    ok, err = gram_close(G1.cpu().numpy()[0], Gb.cpu().numpy().sum(axis=0))
+    assert ok, err
+    for rule in ("mgda", "pcgrad", "cagrad"):
+        out = torch.empty(N, dtype=_tdt(dt), device=DEV)
+        beta = torch.empty(1, K, device=DEV)
+        status = torch.empty(1, dtype=torch.int32, device=DEV)
+        res1.resolve(grads, rule, out, out_weights=beta, out_status=status)
+        torch.cuda.synchronize()
+        _check_against_oracle(w, rule, one, hv, out, beta.cpu().numpy(), status.cpu().numpy(), dt)
+
+
 # ---------------------------------------------------------------------------
 # fused path (BKMOO_FLAG_FUSED): one persistent launch per resolve
 # ---------------------------------------------------------------------------
