@@ -67,8 +67,10 @@ def workload(name):
     if name.startswith("qwen3-8b-") and name.endswith("layers"):
         return inputs.qwen3_8b_layers(int(name[len("qwen3-8b-"):-len("layers")]))
     if name.startswith("sweep-"):
-        _, k, mib = name.split("-")
-        return inputs.sweep(int(k), int(mib))
+        # sweep-K-MiB, or sweep-K-MiB-<n>M for a vector of n million elements
+        parts = name.split("-")
+        n = int(parts[3][:-1]) * 1_000_000 if len(parts) > 3 else 1_000_000_000
+        return inputs.sweep(int(parts[1]), int(parts[2]), n)
     raise SystemExit("unknown workload " + name)
 
 

@@ -248,6 +248,29 @@ int bkmoo_resolve(const void* const* grads, int32_t K, int32_t in_dtype,
                   size_t ws_bytes, void* stream);
 
 /*
+ * bkmoo_resolve_buckets -- bkmoo_resolve for the buckets b_lo .. b_hi-1 of
+ * the plan only.  Algorithm 1 resolves bucket k as soon as the backward pass
+ * has filled it (its interception "when bucket k is full", Figure 4), while
+ * the rest of the backward pass still runs: this entry point lets a caller
+ * resolve each bucket as it completes, on any stream.
+ *
+ * Arguments as in bkmoo_resolve (the whole plan's offsets and workspace),
+ * plus 0 <= b_lo <= b_hi <= n_buckets (else BKMOO_ERR_INVALID; b_lo == b_hi
+ * queues nothing).  Only those buckets' Gram, rule and combination run: the
+ * elements of out_dir, the rows of out_weights / out_status and the
+ * workspace partials of other buckets are not touched, so calls for disjoint
+ * bucket ranges may run concurrently on different streams.  Results are
+ * bit-identical to bkmoo_resolve's for the same buckets.  The workspace
+ * status word is not cleared (other calls may be in flight); device-side
+ * errors are recorded into it.  BKMOO_FLAG_FUSED and p->events are ignored.
+ */
+int bkmoo_resolve_buckets(const void* const* grads, int32_t K, int32_t in_dtype,
+                          const int64_t* offsets, int64_t n_buckets, int64_t b_lo, int64_t b_hi,
+                          int32_t rule, const bkmoo_params* p, void* out_dir, int32_t out_dtype,
+                          float* out_weights, int32_t* out_status, void* ws, size_t ws_bytes,
+                          void* stream);
+
+/*
  * bkmoo_host_staging_size -- device staging bytes bkmoo_resolve_host needs
  * so that every window holds at least max(window_elems, the largest bucket)
  * elements per language.  Host only, pure.  Writes *bytes.

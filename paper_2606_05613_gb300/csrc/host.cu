@@ -58,8 +58,9 @@ LaunchCache& cache() {
   return c;
 }
 
-// Resident CTAs of `fn` on the current device times its SM count.
-cudaError_t persistent_grid(const void* fn, int threads, int* grid) {
+// Resident CTAs of `fn` on the current device times its SM count.  A kernel
+// with dynamic shared memory gets its size limit raised once per device.
+cudaError_t persistent_grid(const void* fn, int threads, int* grid, int dyn_smem = 0) {
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return e;
@@ -76,7 +77,11 @@ cudaError_t persistent_grid(const void* fn, int threads, int* grid) {
   auto jt = c.occ.find(key);
   if (jt == c.occ.end()) {
     int n = 0;
-    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, fn, threads, 0);
+    if (dyn_smem > 48 * 1024) {
+      e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn_smem);
+      if (e != cudaSuccess) return e;
+    }
+    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, fn, threads, dyn_smem);
     if (e != cudaSuccess) return e;
     jt = c.occ.emplace(key, n < 1 ? 1 : n).first;
   }
@@ -86,6 +91,9 @@ cudaError_t persistent_grid(const void* fn, int threads, int* grid) {
 
 const void* gram_fn(int K, int dt) {
   return dt == BKMOO_F32 ? gram_partials_fn_f32(K) : gram_partials_fn_bf16(K);
+}
+const void* gram_staged_fn(int K, int dt) {
+  return dt == BKMOO_F32 ? gram_staged_fn_f32(K) : gram_staged_fn_bf16(K);
 }
 const void* combine_fn(int K, int dti, int dto) {
   return dti == BKMOO_F32 ? combine_fn_f32(K, dto) : combine_fn_bf16(K, dto);
@@ -178,14 +186,17 @@ int launch_gram_pass(const GradPtrs& g, const PlanView& v, cudaStream_t s, bool 
     return BKMOO_ERR_CUDA;
   const int64_t nch = v.c_hi - v.c_lo;
   if (nch <= 0) return BKMOO_OK;
-  const void* fn = gram_fn(v.K, v.in_dtype);
+  const bool staged = v.K >= kGramStagedMinK;
+  const void* fn = staged ? gram_staged_fn(v.K, v.in_dtype) : gram_fn(v.K, v.in_dtype);
+  const int threads = staged ? gram_staged_threads() : kThreads;
+  const int smem = staged ? gram_staged_smem(v.K) : 0;
   int grid = 0;
-  if (persistent_grid(fn, kThreads, &grid) != cudaSuccess) return BKMOO_ERR_CUDA;
+  if (persistent_grid(fn, threads, &grid, smem) != cudaSuccess) return BKMOO_ERR_CUDA;
   if (grid > nch) grid = (int)nch;
   GradPtrs ga = g;
   PlanView va = v;
   void* args[] = {&ga, &va};
-  if (cudaLaunchKernel(fn, dim3(grid), dim3(kThreads), args, 0, s) != cudaSuccess)
+  if (cudaLaunchKernel(fn, dim3(grid), dim3(threads), args, smem, s) != cudaSuccess)
     return BKMOO_ERR_CUDA;
   return BKMOO_OK;
 }
@@ -221,6 +232,29 @@ SolveParams solve_params(int32_t rule, const bkmoo_params& prm) {
   sp.step = prm.step;
   sp.flags = prm.flags;
   return sp;
+}
+
+// Checks shared by bkmoo_resolve and bkmoo_resolve_buckets; fills the
+// effective parameters, the plan view and the gradient pointers.
+int resolve_args(const void* const* grads, int32_t K, int32_t in_dtype, const int64_t* offsets,
+                 int64_t n_buckets, int32_t rule, const bkmoo_params* p, const void* out_dir,
+                 int32_t out_dtype, void* ws, size_t ws_bytes, bkmoo_params* prm, PlanView* v,
+                 GradPtrs* g) {
+  if (rule < BKMOO_MGDA || rule > BKMOO_MEAN || !dtype_ok(out_dtype)) return BKMOO_ERR_INVALID;
+  if (!out_dir || !aligned(out_dir, 16)) return BKMOO_ERR_INVALID;
+  if (p) *prm = *p;
+  else bkmoo_default_params(prm);
+  if (!params_ok(*prm)) return BKMOO_ERR_INVALID;
+  int r = prepare(grads, K, in_dtype, offsets, n_buckets, ws, ws_bytes, v, g);
+  if (r != BKMOO_OK) return r;
+  // out_dir may be exactly one gradient (same dtype); any other overlap is refused.
+  const uintptr_t N = (uintptr_t)offsets[n_buckets];
+  const uintptr_t o0 = (uintptr_t)out_dir, o1 = o0 + N * elem_bytes(out_dtype);
+  for (int k = 0; k < K; ++k) {
+    const uintptr_t g0 = (uintptr_t)grads[k], g1 = g0 + N * elem_bytes(in_dtype);
+    if (o0 < g1 && g0 < o1 && !(o0 == g0 && out_dtype == in_dtype)) return BKMOO_ERR_INVALID;
+  }
+  return BKMOO_OK;
 }
 
 // ---------------------------------------------------------------------------
@@ -370,23 +404,12 @@ int bkmoo_resolve(const void* const* grads, int32_t K, int32_t in_dtype, const i
                   int64_t n_buckets, int32_t rule, const bkmoo_params* p, void* out_dir,
                   int32_t out_dtype, float* out_weights, int32_t* out_status, void* ws,
                   size_t ws_bytes, void* stream) {
-  if (rule < BKMOO_MGDA || rule > BKMOO_MEAN || !dtype_ok(out_dtype)) return BKMOO_ERR_INVALID;
-  if (!out_dir || !aligned(out_dir, 16)) return BKMOO_ERR_INVALID;
   bkmoo_params prm;
-  if (p) prm = *p;
-  else bkmoo_default_params(&prm);
-  if (!params_ok(prm)) return BKMOO_ERR_INVALID;
   PlanView v;
   GradPtrs g;
-  int r = prepare(grads, K, in_dtype, offsets, n_buckets, ws, ws_bytes, &v, &g);
+  int r = resolve_args(grads, K, in_dtype, offsets, n_buckets, rule, p, out_dir, out_dtype, ws,
+                       ws_bytes, &prm, &v, &g);
   if (r != BKMOO_OK) return r;
-  // out_dir may be exactly one gradient (same dtype); any other overlap is refused.
-  const uintptr_t N = (uintptr_t)offsets[n_buckets];
-  const uintptr_t o0 = (uintptr_t)out_dir, o1 = o0 + N * elem_bytes(out_dtype);
-  for (int k = 0; k < K; ++k) {
-    const uintptr_t g0 = (uintptr_t)grads[k], g1 = g0 + N * elem_bytes(in_dtype);
-    if (o0 < g1 && g0 < o1 && !(o0 == g0 && out_dtype == in_dtype)) return BKMOO_ERR_INVALID;
-  }
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   cudaEvent_t* ev = static_cast<cudaEvent_t*>(prm.events);
   const SolveParams sp = solve_params(rule, prm);
@@ -411,6 +434,34 @@ int bkmoo_resolve(const void* const* grads, int32_t K, int32_t in_dtype, const i
   if (r != BKMOO_OK) return r;
   if (ev && cudaEventRecord(ev[3], s) != cudaSuccess) return BKMOO_ERR_CUDA;
   return BKMOO_OK;
+}
+
+int bkmoo_resolve_buckets(const void* const* grads, int32_t K, int32_t in_dtype,
+                          const int64_t* offsets, int64_t n_buckets, int64_t b_lo, int64_t b_hi,
+                          int32_t rule, const bkmoo_params* p, void* out_dir, int32_t out_dtype,
+                          float* out_weights, int32_t* out_status, void* ws, size_t ws_bytes,
+                          void* stream) {
+  bkmoo_params prm;
+  PlanView v;
+  GradPtrs g;
+  int r = resolve_args(grads, K, in_dtype, offsets, n_buckets, rule, p, out_dir, out_dtype, ws,
+                       ws_bytes, &prm, &v, &g);
+  if (r != BKMOO_OK) return r;
+  if (b_lo < 0 || b_hi > n_buckets || b_lo > b_hi) return BKMOO_ERR_INVALID;
+  if (b_lo == b_hi) return BKMOO_OK;
+  v.b_lo = b_lo;
+  v.b_hi = b_hi;
+  int64_t c = 0;
+  for (int64_t b = 0; b < b_lo; ++b) c += (offsets[b + 1] - offsets[b] + v.chunk_elems - 1) / v.chunk_elems;
+  v.c_lo = c;
+  for (int64_t b = b_lo; b < b_hi; ++b) c += (offsets[b + 1] - offsets[b] + v.chunk_elems - 1) / v.chunk_elems;
+  v.c_hi = c;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const SolveParams sp = solve_params(rule, prm);
+  r = launch_gram_pass(g, v, s, false);
+  if (r != BKMOO_OK) return r;
+  if (launch_solve(v, sp, out_weights, out_status, s) != cudaSuccess) return BKMOO_ERR_CUDA;
+  return launch_combine(g, v, out_dir, out_dtype, s);
 }
 
 int bkmoo_host_staging_size(int32_t K, int32_t in_dtype, int32_t out_dtype,

@@ -86,6 +86,10 @@ def load():
         lib.bkmoo_resolve.restype = ctypes.c_int
         lib.bkmoo_resolve.argtypes = [vp, i32, i32, vp, i64, i32, ctypes.POINTER(bkmoo_params),
                                       vp, i32, vp, vp, vp, sz, vp]
+        lib.bkmoo_resolve_buckets.restype = ctypes.c_int
+        lib.bkmoo_resolve_buckets.argtypes = [vp, i32, i32, vp, i64, i64, i64, i32,
+                                              ctypes.POINTER(bkmoo_params), vp, i32, vp, vp, vp,
+                                              sz, vp]
         lib.bkmoo_host_staging_size.restype = ctypes.c_int
         lib.bkmoo_host_staging_size.argtypes = [i32, i32, i32, vp, i64, i64, ctypes.POINTER(sz)]
         lib.bkmoo_resolve_host.restype = ctypes.c_int
@@ -217,6 +221,24 @@ def bkmoo_resolve(grads, offsets, rule, out_dir, ws, params=None, out_weights=No
                                 _stream_handle(stream, grads[0].device)), "bkmoo_resolve")
 
 
+def bkmoo_resolve_buckets(grads, offsets, b_lo, b_hi, rule, out_dir, ws, params=None,
+                          out_weights=None, out_status=None, stream=None):
+    if isinstance(rule, str):
+        rule = RULES[rule]
+    off = _offsets_array(offsets)
+    ptrs = _grad_ptrs(grads)
+    p = params if params is not None else bkmoo_default_params()
+    _check(load().bkmoo_resolve_buckets(ptrs, len(grads), _dtype_code(grads[0]), off.ctypes.data,
+                                        len(off) - 1, b_lo, b_hi, rule, ctypes.byref(p),
+                                        out_dir.data_ptr(), _dtype_code(out_dir),
+                                        out_weights.data_ptr() if out_weights is not None
+                                        else None,
+                                        out_status.data_ptr() if out_status is not None else None,
+                                        ws.data_ptr(), ws.numel() * ws.element_size(),
+                                        _stream_handle(stream, grads[0].device)),
+           "bkmoo_resolve_buckets")
+
+
 def bkmoo_host_staging_size(K: int, in_dtype: int, out_dtype: int, offsets,
                             window_elems: int = 0) -> int:
     off = _offsets_array(offsets)
@@ -289,6 +311,11 @@ class Resolver:
                 stream=None):
         bkmoo_resolve(grads, self.offsets, rule, out_dir, self.ws, params, out_weights,
                       out_status, stream)
+
+    def resolve_buckets(self, grads, b_lo, b_hi, rule, out_dir, params=None, out_weights=None,
+                        out_status=None, stream=None):
+        bkmoo_resolve_buckets(grads, self.offsets, b_lo, b_hi, rule, out_dir, self.ws, params,
+                              out_weights, out_status, stream)
 
     def resolve_host(self, host_grads, rule, host_out, staging, params=None, out_weights=None,
                      out_status=None, stream=None):
