@@ -219,17 +219,6 @@ __device__ __forceinline__ float load_scalar(const void* base, int64_t i) {
 const void* gram_partials_fn_f32(int K);
 const void* gram_partials_fn_bf16(int K);
 
-// Shared-memory-staged Gram-pass kernels (same signature), for K >=
-// kGramStagedMinK; gram_staged_*.cu.
-#ifndef BKMOO_STAGED_MIN_K
-#define BKMOO_STAGED_MIN_K 17
-#endif
-constexpr int kGramStagedMinK = BKMOO_STAGED_MIN_K;
-const void* gram_staged_fn_f32(int K);
-const void* gram_staged_fn_bf16(int K);
-int gram_staged_threads();
-int gram_staged_smem(int K);
-
 // Combine kernels, signature (GradPtrs, PlanView, void* out); combine_*.cu.
 const void* combine_fn_f32(int K, int dtype_out);
 const void* combine_fn_bf16(int K, int dtype_out);

@@ -58,9 +58,8 @@ LaunchCache& cache() {
   return c;
 }
 
-// Resident CTAs of `fn` on the current device times its SM count.  A kernel
-// with dynamic shared memory gets its size limit raised once per device.
-cudaError_t persistent_grid(const void* fn, int threads, int* grid, int dyn_smem = 0) {
+// Resident CTAs of `fn` on the current device times its SM count.
+cudaError_t persistent_grid(const void* fn, int threads, int* grid) {
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return e;
@@ -77,11 +76,7 @@ cudaError_t persistent_grid(const void* fn, int threads, int* grid, int dyn_smem
   auto jt = c.occ.find(key);
   if (jt == c.occ.end()) {
     int n = 0;
-    if (dyn_smem > 48 * 1024) {
-      e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn_smem);
-      if (e != cudaSuccess) return e;
-    }
-    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, fn, threads, dyn_smem);
+    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, fn, threads, 0);
     if (e != cudaSuccess) return e;
     jt = c.occ.emplace(key, n < 1 ? 1 : n).first;
   }
@@ -91,9 +86,6 @@ cudaError_t persistent_grid(const void* fn, int threads, int* grid, int dyn_smem
 
 const void* gram_fn(int K, int dt) {
   return dt == BKMOO_F32 ? gram_partials_fn_f32(K) : gram_partials_fn_bf16(K);
-}
-const void* gram_staged_fn(int K, int dt) {
-  return dt == BKMOO_F32 ? gram_staged_fn_f32(K) : gram_staged_fn_bf16(K);
 }
 const void* combine_fn(int K, int dti, int dto) {
   return dti == BKMOO_F32 ? combine_fn_f32(K, dto) : combine_fn_bf16(K, dto);
@@ -186,17 +178,14 @@ int launch_gram_pass(const GradPtrs& g, const PlanView& v, cudaStream_t s, bool 
     return BKMOO_ERR_CUDA;
   const int64_t nch = v.c_hi - v.c_lo;
   if (nch <= 0) return BKMOO_OK;
-  const bool staged = v.K >= kGramStagedMinK;
-  const void* fn = staged ? gram_staged_fn(v.K, v.in_dtype) : gram_fn(v.K, v.in_dtype);
-  const int threads = staged ? gram_staged_threads() : kThreads;
-  const int smem = staged ? gram_staged_smem(v.K) : 0;
+  const void* fn = gram_fn(v.K, v.in_dtype);
   int grid = 0;
-  if (persistent_grid(fn, threads, &grid, smem) != cudaSuccess) return BKMOO_ERR_CUDA;
+  if (persistent_grid(fn, kThreads, &grid) != cudaSuccess) return BKMOO_ERR_CUDA;
   if (grid > nch) grid = (int)nch;
   GradPtrs ga = g;
   PlanView va = v;
   void* args[] = {&ga, &va};
-  if (cudaLaunchKernel(fn, dim3(grid), dim3(threads), args, smem, s) != cudaSuccess)
+  if (cudaLaunchKernel(fn, dim3(grid), dim3(kThreads), args, 0, s) != cudaSuccess)
     return BKMOO_ERR_CUDA;
   return BKMOO_OK;
 }
