@@ -948,8 +948,8 @@ __device__ void cagrad_refine(const double* G, const double (&b)[K], double rho,
   for (int i = 0; i < K; ++i) w[i] *= corr;
 }
 
-// Exact CAGrad for 1 <= K <= 5.  False if the check fails or a case that
-// needs the minimum-norm candidate (0 possibly in the hull) comes up.
+// Exact CAGrad for 1 <= K <= 5.  False if no candidate passes the
+// optimality check (e.g. the minimum of F at g_w = 0).
 template <int K>
 __device__ bool cagrad_fast(const double* G, const float* Gf, double c, int lane,
                             double* beta_out) {
@@ -971,10 +971,11 @@ __device__ bool cagrad_fast(const double* G, const float* Gf, double c, int lane
       for (int k = 0; k < K; ++k) beta_out[k] = 1.0 / K;
     return true;
   }
-  bool all_pos = true;
-#pragma unroll
-  for (int i = 0; i < K; ++i) all_pos = all_pos && (b[i] > 0.0);
-  if (!all_pos) return false;  // 0 may lie in the hull: serial path
+  // No sign condition on b: when 0 may lie in the hull (some b_k <= 0) the
+  // minimiser still has g_w != 0 unless F's minimum sits at the kink
+  // g_w = 0; the optimality check below certifies the candidate either way
+  // (F is convex and differentiable wherever g_w != 0), and a candidate that
+  // fails it goes to the serial path.
   const double rho = c * sqrt_nr(g0sq);
   float Ginv[K][K], w32[K];
   const unsigned mask = (unsigned)lane + 1u;
@@ -1313,7 +1314,8 @@ __device__ bool cagrad_active_warp(int K, const double* G, const float* Gf, doub
     if (act) beta_out[lane] = 1.0 / K;
     return true;
   }
-  if (!__all_sync(0xffffffffu, !act || bd > 0.0)) return false;  // 0 may lie in the hull
+  // (no sign condition on b: the final optimality check certifies the
+  // result, see cagrad_fast)
   const double rho = c * sqrt_nr(g0sq);
   const float rhof = (float)rho, bf = (float)bd;
   const float Fv = act ? bf + rhof * sqrtf(fmaxf(Gf[lane * K + lane], 0.0f)) : INFINITY;

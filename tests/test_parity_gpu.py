@@ -128,6 +128,17 @@ def test_every_k_mgda_and_cagrad_f32(K):
         _check_against_oracle(w, rule, off, hv, out, beta, status, "f32")
 
 
+@pytest.mark.parametrize("K", [2, 3, 5, 6, 8, 12, 16])
+def test_opposed_language_cagrad_and_mgda(K):
+    """One language sign-flipped in every bucket over a strong shared part:
+    <g_k, g0> < 0 for that language, the case where 0 may lie in the hull
+    (Eq. 4's dual is then minimised away from its kink in general)."""
+    w = _workload(K, "f32", [200000, 9, 77777], 90000, seed=70 + K, rho=(0.6, 0.95), flip=1.0)
+    for rule in ("cagrad", "mgda"):
+        off, hv, out, beta, status, _ = _run(w, rule, "f32")
+        _check_against_oracle(w, rule, off, hv, out, beta, status, "f32")
+
+
 @pytest.mark.parametrize("rule", ["mgda", "pcgrad", "cagrad"])
 def test_in_place_equals_out_of_place(rule):
     w = _workload(4, "bf16", RAGGED, 180000, seed=3)
