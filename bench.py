@@ -164,6 +164,13 @@ class ClockSampler:
                 "reasons": reasons, "samples": len(rows)}
 
 
+def base_config(w, off, rule):
+    """The workload description both arms print."""
+    return {"workload": w.name, "K": w.K, "grad_dtype": w.dtype, "out_dtype": w.dtype,
+            "rule": rule, "n_elems_per_language": int(off[-1]), "n_buckets": len(off) - 1,
+            "bucket_bytes": w.bucket_bytes}
+
+
 def reduce_over_ranks(ms_step, grad_bytes, device):
     """Whole-job throughput: the gradient bytes of all ranks over the slowest
     rank's time per step.  Returns (max ms per step, GB/s).  One rank: no
@@ -180,7 +187,7 @@ def reduce_over_ranks(ms_step, grad_bytes, device):
     return ms, float(u.item()) / (ms * 1e-3) / GB
 
 
-def cpu_baseline(w, offsets, seconds, n_threads=0):
+def cpu_baseline(w, offsets, seconds, n_threads=0, rule="mgda"):
     """The oracle, as it stands, on a bounded sample of the workload's
     buckets (host-generated with the same generator), repeated until about
     `seconds` of wall time; returns (GB/s of gradient bytes, cores, sample)."""
@@ -211,14 +218,15 @@ def cpu_baseline(w, offsets, seconds, n_threads=0):
     t0 = time.perf_counter()
     passes = 0
     while True:
-        orc.resolve(hv, np.array(sub_off, dtype=np.int64), orc.MGDA, n_threads=cores)
+        orc.resolve(hv, np.array(sub_off, dtype=np.int64), getattr(orc, rule.upper()),
+                    n_threads=cores)
         passes += 1
         if time.perf_counter() - t0 >= seconds:
             break
     dt = time.perf_counter() - t0
     grad_bytes = w.K * sub_off[-1] * w.elem_bytes * passes
-    sample = ("%d of %d buckets (%d elements per language), %d passes, MGDA exact"
-              % (len(picks), B, sub_off[-1], passes))
+    sample = ("%d of %d buckets (%d elements per language), %d passes, %s"
+              % (len(picks), B, sub_off[-1], passes, rule))
     return grad_bytes / dt / GB, cores, sample, dt / passes
 
 
@@ -258,12 +266,12 @@ def run_reference(a):
     off = orc.plan(w.param_sizes, w.elem_bytes, w.bucket_bytes)
     # each step: one oracle pass over a sample of one bucket per core
     for _ in range(a.warmup):
-        cpu_baseline(w, off, 0.0)
+        cpu_baseline(w, off, 0.0, rule=a.rule)
     vals, times = [], []
     cores = orc.max_threads()
     sample = ""
     for _ in range(a.steps):
-        v, cores, sample, t = cpu_baseline(w, off, 0.0)
+        v, cores, sample, t = cpu_baseline(w, off, 0.0, rule=a.rule)
         vals.append(v)
         times.append(t)
     v = sum(vals) / len(vals)
@@ -272,9 +280,9 @@ def run_reference(a):
         "value": v, "unit": "GB/s", "n_gpus": a.gpus, "steps": a.steps, "warmup": a.warmup,
         "ms_per_step": 1e3 * sum(times) / len(times), "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-        "config": {"workload": w.name, "K": w.K, "grad_dtype": w.dtype, "rule": "mgda",
-                   "n_elems": w.n_elems, "n_buckets": len(off) - 1,
-                   "note": "fp64 CPU oracle (plain C, OpenMP over buckets) on a sample"},
+        "config": dict(base_config(w, off, a.rule),
+                       parallelism="host cores (OpenMP over buckets)",
+                       path="fp64 CPU oracle (plain C) on a sample of buckets"),
         "cpu_baseline": {"value": v, "unit": "GB/s", "cores": cores, "kind": "oracle",
                          "sample": sample},
         "e2e": {"value": v, "unit": "GB/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
@@ -395,13 +403,12 @@ def main():
         "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "f32" if w.dtype == "f32" else "bf16",
         "data": "synthetic",
-        "config": {"workload": w.name, "K": w.K, "grad_dtype": w.dtype, "out_dtype": w.dtype,
-                   "rule": a.rule, "n_elems_per_language": N, "n_buckets": B,
-                   "bucket_bytes": w.bucket_bytes, "l2": "inputs (%.1f GB) >> L2, no flush"
-                   % (grad_bytes / GB), "parallelism": "replicas" if world > 1 else "1 GPU",
-                   "path": ("fused: one persistent launch per step, combination re-reads "
-                            "each bucket from L2" if fused else
-                            "gram -> solve -> combine (3 launches)")},
+        "config": dict(base_config(w, off, a.rule),
+                       l2="inputs (%.1f GB) >> L2, no flush" % (grad_bytes / GB),
+                       parallelism="replicas" if world > 1 else "1 GPU",
+                       path=("fused: one persistent launch per step, combination re-reads "
+                             "each bucket from L2" if fused else
+                             "gram -> solve -> combine (3 launches)")),
         "roofline": roofline,
         "step_roofline": {"bytes_2k1": step_bytes_2k1, "bytes_k1": step_bytes_k1,
                           "frac_2k1_of_measured": step_bytes_2k1 / (ms_step * 1e-3) / GB / peak,
@@ -419,7 +426,7 @@ def main():
     if rank == 0 and world == 1 and not a.no_cpu_baseline:
         del grads
         torch.cuda.empty_cache()
-        v, cores, sample, _ = cpu_baseline(w, off, a.cpu_seconds)
+        v, cores, sample, _ = cpu_baseline(w, off, a.cpu_seconds, rule=a.rule)
         line["cpu_baseline"] = {"value": v, "unit": "GB/s", "cores": cores, "kind": "oracle",
                                 "sample": sample}
     if rank == 0:

@@ -77,7 +77,35 @@ __global__ void __launch_bounds__(kThreads) combine_kernel(const GradPtrs g, con
     if (ve < vs) ve = vs;
     const int nv = (int)((ve - vs) / EPV);
 
-    for (int i = threadIdx.x; i < nv; i += kThreads) {
+    int i = threadIdx.x;
+    // K >= 9: two vectors per thread in flight (measured 8 % faster at K = 16;
+    // no change at K = 4 and 8, where the occupancy already hides the latency)
+    if (K >= 9) {
+      for (; i + kThreads < nv; i += 2 * kThreads) {
+        const int64_t el0 = vs + (int64_t)i * EPV, el1 = el0 + (int64_t)kThreads * EPV;
+        uint4 r0[K], r1[K];
+#pragma unroll
+        for (int k = 0; k < K; ++k) {
+          r0[k] = ld16_cs(static_cast<const char*>(g.p[k]) + el0 * IB);
+          r1[k] = ld16_cs(static_cast<const char*>(g.p[k]) + el1 * IB);
+        }
+        float y0[EPV], y1[EPV];
+#pragma unroll
+        for (int q = 0; q < EPV; ++q) {
+          float t0 = 0.0f, t1 = 0.0f;
+#pragma unroll
+          for (int k = 0; k < K; ++k) {
+            t0 = fmaf(beta[k], vec_elem<DTI>(r0[k], q), t0);
+            t1 = fmaf(beta[k], vec_elem<DTI>(r1[k], q), t1);
+          }
+          y0[q] = t0;
+          y1[q] = t1;
+        }
+        store_out<DTO>(out, el0, y0, EPV);
+        store_out<DTO>(out, el1, y1, EPV);
+      }
+    }
+    for (; i < nv; i += kThreads) {
       const int64_t el = vs + (int64_t)i * EPV;
       uint4 r[K];
 #pragma unroll
