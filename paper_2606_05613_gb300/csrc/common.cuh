@@ -219,6 +219,13 @@ __device__ __forceinline__ float load_scalar(const void* base, int64_t i) {
 const void* gram_partials_fn_f32(int K);
 const void* gram_partials_fn_bf16(int K);
 
+// Gram-pass kernels with a per-thread shared-memory prefetch (same signature,
+// kThreads threads, gram_prefetch_smem(K) bytes of dynamic shared memory) for
+// K >= gram_prefetch_min_k(); nullptr below; gram_prefetch.cu.
+const void* gram_prefetch_fn(int K, int dt);
+int gram_prefetch_smem(int K);
+int gram_prefetch_min_k();
+
 // Combine kernels, signature (GradPtrs, PlanView, void* out); combine_*.cu.
 const void* combine_fn_f32(int K, int dtype_out);
 const void* combine_fn_bf16(int K, int dtype_out);

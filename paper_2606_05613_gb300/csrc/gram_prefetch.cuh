@@ -1,0 +1,170 @@
+// Gram pass for large K with a per-thread prefetch into shared memory.
+//
+// At K >= 12 a thread's K(K+1)/2 fp32 accumulators (136 at K = 16) leave
+// room for 8 warps per SM, and a thread that loads its K vectors into
+// registers and then computes keeps one load batch in flight at a time.
+// Here each thread copies its next vector sets into its own shared-memory
+// slots with cp.async (16-byte LDGSTS, no register cost), S stages ahead,
+// and computes from the oldest stage; a thread reads only slots it wrote
+// itself, so cp.async.wait_group is the only synchronisation.  The chunks,
+// the per-thread element order, the fp32 sums and the fixed reduction are
+// those of gram_partials_kernel (gram_impl.cuh), so the partials are
+// bit-identical to it.
+#pragma once
+
+#include "gram_impl.cuh"
+
+namespace bkmoo {
+
+constexpr int kPrefetchMinK = 12;
+constexpr int kPrefetchStages = 3;
+
+__host__ __device__ constexpr int prefetch_smem_bytes(int K) {
+  return kPrefetchStages * K * kThreads * 16;
+}
+
+__device__ __forceinline__ void cp_async16(void* smem_dst, const void* src) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(
+                   (uint32_t)__cvta_generic_to_shared(smem_dst)),
+               "l"(src)
+               : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() {
+  asm volatile("cp.async.commit_group;" ::: "memory");
+}
+template <int N>
+__device__ __forceinline__ void cp_async_wait() {
+  asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
+}
+
+// find_bucket with, after the hint, a guess that is exact when the buckets
+// from the hint on have the hint's chunk count (one tensor cut into equal
+// buckets): with one CTA per SM a CTA's next chunk lies about 152 chunks on,
+// many small buckets away, and the binary search's dependent loads sit on
+// the path of the copies this kernel issues.  (The other kernels keep the
+// plain search: the guess costs them registers and occupancy.)
+__device__ __forceinline__ int64_t find_bucket_guess(const int64_t* cp, int64_t B, int64_t w,
+                                                     int64_t hint) {
+  if (hint < B && cp[hint] <= w) {
+    const int64_t c0 = cp[hint], c1 = cp[hint + 1];
+    if (w < c1) return hint;
+    const int64_t g = hint + (w - c0) / (c1 > c0 ? c1 - c0 : 1);
+    if (g < B && cp[g] <= w && w < cp[g + 1]) return g;
+  }
+  return find_bucket(cp, B, w, hint);
+}
+
+// This thread's sequence of 16-byte positions: chunk w = c_lo + blockIdx.x,
+// + gridDim.x, ...; within a chunk the vectors i = t, t + 256, ... < nv.
+template <int EPV>
+struct VecCursor {
+  int64_t w, b, vs;
+  int nv, i;
+  __device__ void settle(const PlanView& v) {
+    while (w < v.c_hi) {
+      b = find_bucket_guess(v.chunk_prefix, v.n_buckets, w, b);
+      const int64_t be = v.offsets[b + 1];
+      const int64_t s = v.offsets[b] + (w - v.chunk_prefix[b]) * v.chunk_elems;
+      const int64_t e = min(s + v.chunk_elems, be);
+      int64_t a = (s + EPV - 1) / EPV * EPV;
+      if (a > e) a = e;
+      int64_t z = e / EPV * EPV;
+      if (z < a) z = a;
+      vs = a;
+      nv = (int)((z - a) / EPV);
+      if (i < nv) return;
+      w += gridDim.x;
+      i = threadIdx.x;
+    }
+  }
+  __device__ void begin(const PlanView& v) {
+    w = v.c_lo + blockIdx.x;
+    b = v.b_lo;
+    i = threadIdx.x;
+    settle(v);
+  }
+  __device__ bool more(const PlanView& v) const { return w < v.c_hi; }
+  __device__ void next(const PlanView& v) {
+    i += kThreads;
+    if (i >= nv) settle(v);
+  }
+};
+
+template <int K, int DT>
+__global__ void __launch_bounds__(kThreads) gram_prefetch_kernel(const GradPtrs g,
+                                                                 const PlanView v) {
+  constexpr int P = tri(K);
+  constexpr int EPV = elems_per_vec(DT);
+  constexpr int IB = 16 / EPV;
+  constexpr int S = kPrefetchStages;
+  extern __shared__ __align__(16) unsigned char pf_smem[];
+  __shared__ float red[kWarps][P];
+  // slot (stage s, gradient k) of thread t
+  uint4* slots = reinterpret_cast<uint4*>(pf_smem);
+  auto slot = [&](int s, int k) -> uint4* { return slots + ((s * K + k) * kThreads + threadIdx.x); };
+
+  if (!header_ok(v)) {
+    if (blockIdx.x == 0 && threadIdx.x == 0) record_error(v.hdr, BKMOO_ERR_WORKSPACE);
+    return;
+  }
+  // the producer cursor runs S - 1 positions ahead of the consumer
+  VecCursor<EPV> pc;
+  pc.begin(v);
+  int issued = 0;
+  auto issue = [&]() {
+    const int s = issued % S;
+    if (pc.more(v)) {
+      const int64_t off = (pc.vs + (int64_t)pc.i * EPV) * IB;
+#pragma unroll
+      for (int k = 0; k < K; ++k) cp_async16(slot(s, k), static_cast<const char*>(g.p[k]) + off);
+      pc.next(v);
+    }
+    cp_async_commit();   // empty groups keep the group count in step
+    ++issued;
+  };
+#pragma unroll
+  for (int j = 0; j < S - 1; ++j) issue();
+
+  int consumed = 0;
+  int64_t b = v.b_lo;
+  for (int64_t w = v.c_lo + blockIdx.x; w < v.c_hi; w += gridDim.x) {
+    b = find_bucket_guess(v.chunk_prefix, v.n_buckets, w, b);
+    const int64_t be = v.offsets[b + 1];
+    const int64_t s0 = v.offsets[b] + (w - v.chunk_prefix[b]) * v.chunk_elems;
+    const int64_t e = min(s0 + v.chunk_elems, be);
+    int64_t vs = (s0 + EPV - 1) / EPV * EPV;
+    if (vs > e) vs = e;
+    int64_t ve = e / EPV * EPV;
+    if (ve < vs) ve = vs;
+    const int nv = (int)((ve - vs) / EPV);
+
+    float acc[P];
+#pragma unroll
+    for (int p = 0; p < P; ++p) acc[p] = 0.0f;
+    for (int i = threadIdx.x; i < nv; i += kThreads) {
+      issue();                       // position consumed + S - 1
+      cp_async_wait<S - 1>();        // the oldest group (this position) has landed
+      const int s = consumed % S;
+      uint4 r[K];
+#pragma unroll
+      for (int k = 0; k < K; ++k) r[k] = *slot(s, k);
+      gram_accumulate<K, DT>(acc, r);
+      ++consumed;
+    }
+    const int nh = (int)(vs - s0), nt = (int)(e - ve);
+    if ((int)threadIdx.x < nh + nt) {
+      const int64_t idx = (int)threadIdx.x < nh ? s0 + threadIdx.x : ve + (threadIdx.x - nh);
+      gram_accumulate_scalar<K, DT>(acc, g, idx);
+    }
+    cta_reduce_store<P>(acc, red, v.partials + w * P);
+  }
+  cp_async_wait<0>();
+}
+
+#define BKMOO_GRAM_PREFETCH_TABLE(DT)                                                       \
+  static const void* const kGramPrefetchTable[kMaxK - kPrefetchMinK + 1] = {                \
+      (const void*)gram_prefetch_kernel<12, DT>, (const void*)gram_prefetch_kernel<13, DT>, \
+      (const void*)gram_prefetch_kernel<14, DT>, (const void*)gram_prefetch_kernel<15, DT>, \
+      (const void*)gram_prefetch_kernel<16, DT>}
+
+}  // namespace bkmoo

@@ -58,8 +58,9 @@ LaunchCache& cache() {
   return c;
 }
 
-// Resident CTAs of `fn` on the current device times its SM count.
-cudaError_t persistent_grid(const void* fn, int threads, int* grid) {
+// Resident CTAs of `fn` on the current device times its SM count.  A kernel
+// with more than 48 KiB of dynamic shared memory gets its limit raised once.
+cudaError_t persistent_grid(const void* fn, int threads, int* grid, int dyn_smem = 0) {
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return e;
@@ -76,7 +77,11 @@ cudaError_t persistent_grid(const void* fn, int threads, int* grid) {
   auto jt = c.occ.find(key);
   if (jt == c.occ.end()) {
     int n = 0;
-    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, fn, threads, 0);
+    if (dyn_smem > 48 * 1024) {
+      e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn_smem);
+      if (e != cudaSuccess) return e;
+    }
+    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, fn, threads, dyn_smem);
     if (e != cudaSuccess) return e;
     jt = c.occ.emplace(key, n < 1 ? 1 : n).first;
   }
@@ -178,14 +183,17 @@ int launch_gram_pass(const GradPtrs& g, const PlanView& v, cudaStream_t s, bool 
     return BKMOO_ERR_CUDA;
   const int64_t nch = v.c_hi - v.c_lo;
   if (nch <= 0) return BKMOO_OK;
-  const void* fn = gram_fn(v.K, v.in_dtype);
+  // large K: the variant that prefetches into shared memory (gram_prefetch.cu)
+  const bool pf = v.K >= gram_prefetch_min_k();
+  const void* fn = pf ? gram_prefetch_fn(v.K, v.in_dtype) : gram_fn(v.K, v.in_dtype);
+  const int smem = pf ? gram_prefetch_smem(v.K) : 0;
   int grid = 0;
-  if (persistent_grid(fn, kThreads, &grid) != cudaSuccess) return BKMOO_ERR_CUDA;
+  if (persistent_grid(fn, kThreads, &grid, smem) != cudaSuccess) return BKMOO_ERR_CUDA;
   if (grid > nch) grid = (int)nch;
   GradPtrs ga = g;
   PlanView va = v;
   void* args[] = {&ga, &va};
-  if (cudaLaunchKernel(fn, dim3(grid), dim3(kThreads), args, 0, s) != cudaSuccess)
+  if (cudaLaunchKernel(fn, dim3(grid), dim3(kThreads), args, smem, s) != cudaSuccess)
     return BKMOO_ERR_CUDA;
   return BKMOO_OK;
 }

@@ -167,16 +167,22 @@ extern "C" int bkmoo_gram_noalloc(const void* const* grads, int32_t K, int32_t i
   std::memset(&g, 0, sizeof g);
   for (int k = 0; k < K; ++k) g.p[k] = grads[k];
 
-  const void* fn = in_dtype == BKMOO_F32 ? gram_partials_fn_f32(K) : gram_partials_fn_bf16(K);
+  // the same Gram-pass kernel as bkmoo_gram (the prefetching variant for large K)
+  const bool pf = K >= gram_prefetch_min_k();
+  const void* fn = pf ? gram_prefetch_fn(K, in_dtype)
+                      : (in_dtype == BKMOO_F32 ? gram_partials_fn_f32(K) : gram_partials_fn_bf16(K));
+  const int smem = pf ? gram_prefetch_smem(K) : 0;
   int dev = 0, sms = 0, per_sm = 0;
   if (cudaGetDevice(&dev) != cudaSuccess ||
       cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess ||
-      cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, fn, kThreads, 0) != cudaSuccess)
+      (smem > 48 * 1024 &&
+       cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) != cudaSuccess) ||
+      cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, fn, kThreads, smem) != cudaSuccess)
     return BKMOO_ERR_CUDA;
   int64_t grid = (int64_t)sms * (per_sm < 1 ? 1 : per_sm);
   if (grid > nch) grid = nch;
   void* args[] = {&g, &v};
-  if (cudaLaunchKernel(fn, dim3((unsigned)grid), dim3(kThreads), args, 0, s) != cudaSuccess)
+  if (cudaLaunchKernel(fn, dim3((unsigned)grid), dim3(kThreads), args, smem, s) != cudaSuccess)
     return BKMOO_ERR_CUDA;
   if (launch_gram_finalize(v, out_gram, s) != cudaSuccess) return BKMOO_ERR_CUDA;
   return BKMOO_OK;
