@@ -226,6 +226,16 @@ const void* gram_prefetch_fn(int K, int dt);
 int gram_prefetch_smem(int K);
 int gram_prefetch_min_k();
 
+// Combine kernels with a per-thread shared-memory prefetch (same signature,
+// combine_prefetch_smem(K) bytes of dynamic shared memory), K <= 8;
+// combine_prefetch.cu.  Measured 2-6.5 % faster than combine_kernel for
+// K = 2..8 (GB300); combine_kernel serves K >= 9.
+#ifndef BKMOO_COMBINE_PREFETCH
+#define BKMOO_COMBINE_PREFETCH 1
+#endif
+const void* combine_prefetch_fn(int K, int dti, int dto);
+int combine_prefetch_smem(int K);
+
 // Combine kernels, signature (GradPtrs, PlanView, void* out); combine_*.cu.
 const void* combine_fn_f32(int K, int dtype_out);
 const void* combine_fn_bf16(int K, int dtype_out);

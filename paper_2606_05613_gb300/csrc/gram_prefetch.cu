@@ -1,4 +1,5 @@
-// Gram-pass kernels with a per-thread shared-memory prefetch, K = 12..16.
+// Gram-pass kernels with a per-thread shared-memory prefetch (used for K >=
+// kPrefetchMinK).
 #include "gram_prefetch.cuh"
 
 namespace bkmoo {
@@ -12,8 +13,7 @@ BKMOO_GRAM_PREFETCH_TABLE(BKMOO_BF16);
 }  // namespace bf
 const void* gram_prefetch_fn(int K, int dt) {
   if (K < kPrefetchMinK || K > kMaxK) return nullptr;
-  return dt == BKMOO_F32 ? kGramPrefetchTable[K - kPrefetchMinK]
-                         : bf::kGramPrefetchTable[K - kPrefetchMinK];
+  return dt == BKMOO_F32 ? kGramPrefetchTable[K - 1] : bf::kGramPrefetchTable[K - 1];
 }
 int gram_prefetch_smem(int K) { return prefetch_smem_bytes(K); }
 int gram_prefetch_min_k() { return kPrefetchMinK; }

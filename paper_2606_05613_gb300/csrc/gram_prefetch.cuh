@@ -16,7 +16,10 @@
 
 namespace bkmoo {
 
-constexpr int kPrefetchMinK = 12;
+#ifndef BKMOO_GRAM_PREFETCH_MIN_K
+#define BKMOO_GRAM_PREFETCH_MIN_K 12
+#endif
+constexpr int kPrefetchMinK = BKMOO_GRAM_PREFETCH_MIN_K;
 constexpr int kPrefetchStages = 3;
 
 __host__ __device__ constexpr int prefetch_smem_bytes(int K) {
@@ -162,9 +165,14 @@ __global__ void __launch_bounds__(kThreads) gram_prefetch_kernel(const GradPtrs 
 }
 
 #define BKMOO_GRAM_PREFETCH_TABLE(DT)                                                       \
-  static const void* const kGramPrefetchTable[kMaxK - kPrefetchMinK + 1] = {                \
-      (const void*)gram_prefetch_kernel<12, DT>, (const void*)gram_prefetch_kernel<13, DT>, \
-      (const void*)gram_prefetch_kernel<14, DT>, (const void*)gram_prefetch_kernel<15, DT>, \
-      (const void*)gram_prefetch_kernel<16, DT>}
+  static const void* const kGramPrefetchTable[kMaxK] = {                                    \
+      (const void*)gram_prefetch_kernel<1, DT>,  (const void*)gram_prefetch_kernel<2, DT>,  \
+      (const void*)gram_prefetch_kernel<3, DT>,  (const void*)gram_prefetch_kernel<4, DT>,  \
+      (const void*)gram_prefetch_kernel<5, DT>,  (const void*)gram_prefetch_kernel<6, DT>,  \
+      (const void*)gram_prefetch_kernel<7, DT>,  (const void*)gram_prefetch_kernel<8, DT>,  \
+      (const void*)gram_prefetch_kernel<9, DT>,  (const void*)gram_prefetch_kernel<10, DT>, \
+      (const void*)gram_prefetch_kernel<11, DT>, (const void*)gram_prefetch_kernel<12, DT>, \
+      (const void*)gram_prefetch_kernel<13, DT>, (const void*)gram_prefetch_kernel<14, DT>, \
+      (const void*)gram_prefetch_kernel<15, DT>, (const void*)gram_prefetch_kernel<16, DT>}
 
 }  // namespace bkmoo

@@ -59,7 +59,8 @@ LaunchCache& cache() {
 }
 
 // Resident CTAs of `fn` on the current device times its SM count.  A kernel
-// with more than 48 KiB of dynamic shared memory gets its limit raised once.
+// with dynamic shared memory gets its limit raised to that size once (the
+// default limit of 48 KiB counts static and dynamic shared memory together).
 cudaError_t persistent_grid(const void* fn, int threads, int* grid, int dyn_smem = 0) {
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
@@ -77,7 +78,7 @@ cudaError_t persistent_grid(const void* fn, int threads, int* grid, int dyn_smem
   auto jt = c.occ.find(key);
   if (jt == c.occ.end()) {
     int n = 0;
-    if (dyn_smem > 48 * 1024) {
+    if (dyn_smem > 0) {
       e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn_smem);
       if (e != cudaSuccess) return e;
     }
@@ -202,15 +203,18 @@ int launch_combine(const GradPtrs& g, const PlanView& v, void* out, int32_t out_
                    cudaStream_t s) {
   const int64_t nch = v.c_hi - v.c_lo;
   if (nch <= 0) return BKMOO_OK;
-  const void* fn = combine_fn(v.K, v.in_dtype, out_dtype);
+  const bool pf = BKMOO_COMBINE_PREFETCH && v.K <= 8;
+  const void* fn = pf ? combine_prefetch_fn(v.K, v.in_dtype, out_dtype)
+                      : combine_fn(v.K, v.in_dtype, out_dtype);
+  const int smem = pf ? combine_prefetch_smem(v.K) : 0;
   int grid = 0;
-  if (persistent_grid(fn, kThreads, &grid) != cudaSuccess) return BKMOO_ERR_CUDA;
+  if (persistent_grid(fn, kThreads, &grid, smem) != cudaSuccess) return BKMOO_ERR_CUDA;
   if (grid > nch) grid = (int)nch;
   PlanView va = v;
   GradPtrs ga = g;
   void* outp = out;
   void* args[] = {&ga, &va, &outp};
-  if (cudaLaunchKernel(fn, dim3(grid), dim3(kThreads), args, 0, s) != cudaSuccess)
+  if (cudaLaunchKernel(fn, dim3(grid), dim3(kThreads), args, smem, s) != cudaSuccess)
     return BKMOO_ERR_CUDA;
   return BKMOO_OK;
 }

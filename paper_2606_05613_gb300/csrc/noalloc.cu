@@ -175,7 +175,7 @@ extern "C" int bkmoo_gram_noalloc(const void* const* grads, int32_t K, int32_t i
   int dev = 0, sms = 0, per_sm = 0;
   if (cudaGetDevice(&dev) != cudaSuccess ||
       cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess ||
-      (smem > 48 * 1024 &&
+      (smem > 0 &&
        cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) != cudaSuccess) ||
       cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, fn, kThreads, smem) != cudaSuccess)
     return BKMOO_ERR_CUDA;
