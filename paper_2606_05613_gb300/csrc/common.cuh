@@ -242,9 +242,11 @@ const void* combine_fn_bf16(int K, int dtype_out);
 
 // Fused kernels, signature (GradPtrs, FusedView, SolveParams, void* out); fused_*.cu.
 const void* fused_fn_f32_k1_4(int K, int dtype_out);
-const void* fused_fn_f32_k5_8(int K, int dtype_out);
+const void* fused_fn_f32_k5_6(int K, int dtype_out);
+const void* fused_fn_f32_k7_8(int K, int dtype_out);
 const void* fused_fn_bf16_k1_4(int K, int dtype_out);
-const void* fused_fn_bf16_k5_8(int K, int dtype_out);
+const void* fused_fn_bf16_k5_6(int K, int dtype_out);
+const void* fused_fn_bf16_k7_8(int K, int dtype_out);
 
 // solve.cu
 cudaError_t launch_solve(const PlanView& v, const SolveParams& p, float* out_weights,

@@ -452,10 +452,13 @@ __global__ void __launch_bounds__(kThreads, FusedMinBlocks<K>::value)
   {(const void*)fused_resolve_kernel<K, DTI, BKMOO_F32>,                      \
    (const void*)fused_resolve_kernel<K, DTI, BKMOO_BF16>}
 
-// Eight values of K per translation unit (compiled in parallel).
+// A few values of K per translation unit (compiled in parallel).
 #define BKMOO_FUSED_TABLE4(DTI, K0)                                                        \
   static const void* const kFusedTable[4][2] = {                                           \
       BKMOO_FUSED_ROW(K0 + 0, DTI), BKMOO_FUSED_ROW(K0 + 1, DTI),                          \
       BKMOO_FUSED_ROW(K0 + 2, DTI), BKMOO_FUSED_ROW(K0 + 3, DTI)}
+#define BKMOO_FUSED_TABLE2(DTI, K0)                                                        \
+  static const void* const kFusedTable[2][2] = {BKMOO_FUSED_ROW(K0 + 0, DTI),               \
+                                                BKMOO_FUSED_ROW(K0 + 1, DTI)}
 
 }  // namespace bkmoo

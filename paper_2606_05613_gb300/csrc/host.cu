@@ -97,8 +97,11 @@ const void* combine_fn(int K, int dti, int dto) {
   return dti == BKMOO_F32 ? combine_fn_f32(K, dto) : combine_fn_bf16(K, dto);
 }
 const void* fused_fn(int K, int dti, int dto) {
-  if (dti == BKMOO_F32) return K <= 4 ? fused_fn_f32_k1_4(K, dto) : fused_fn_f32_k5_8(K, dto);
-  return K <= 4 ? fused_fn_bf16_k1_4(K, dto) : fused_fn_bf16_k5_8(K, dto);
+  if (dti == BKMOO_F32)
+    return K <= 4 ? fused_fn_f32_k1_4(K, dto)
+                  : (K <= 6 ? fused_fn_f32_k5_6(K, dto) : fused_fn_f32_k7_8(K, dto));
+  return K <= 4 ? fused_fn_bf16_k1_4(K, dto)
+                : (K <= 6 ? fused_fn_bf16_k5_6(K, dto) : fused_fn_bf16_k7_8(K, dto));
 }
 
 // The fused path: one cooperative (co-resident) launch; the last CTA solves.
