@@ -210,3 +210,28 @@ def test_resolve_host_rejects_bad_arguments_without_launch():
     q = bk.bkmoo_default_params()
     q.cagrad_c = -0.5
     assert call(p=ctypes.byref(q)) == bk.BKMOO_ERR_INVALID
+
+
+def test_resolve_buckets_rejects_bad_ranges_without_launch():
+    """bkmoo_resolve_buckets checks its bucket range before any CUDA call;
+    an empty range queues nothing (fake, aligned addresses)."""
+    lib = bk.load()
+    off = np.array([0, 1000, 2500, 4000], dtype=np.int64)
+    base = 1 << 40
+    grads = (ctypes.c_void_p * 2)(base, base + (1 << 20))
+    ws = ctypes.c_void_p(base + (1 << 30))
+    out = ctypes.c_void_p(base + (1 << 31))
+    p = bk.bkmoo_default_params()
+
+    def call(lo, hi, **kw):
+        a = dict(wsb=1 << 30)
+        a.update(kw)
+        return lib.bkmoo_resolve_buckets(grads, 2, 0, off.ctypes.data, 3, lo, hi, 0,
+                                         ctypes.byref(p), out, 0, None, None, ws, a["wsb"],
+                                         None)
+
+    assert call(-1, 2) == bk.BKMOO_ERR_INVALID
+    assert call(0, 4) == bk.BKMOO_ERR_INVALID
+    assert call(2, 1) == bk.BKMOO_ERR_INVALID
+    assert call(1, 1) == bk.BKMOO_OK            # empty range: nothing queued
+    assert call(0, 3, wsb=64) == bk.BKMOO_ERR_WORKSPACE
