@@ -56,13 +56,25 @@ constexpr double kPivot = 1e-13;   // smallest pivot of a non-singular system
 // partial reduction
 // ---------------------------------------------------------------------------
 
+// Lane p sums entry p of the bucket's chunk partials in a fixed order: eight
+// interleaved fp64 running sums (chunk c0 + 8m + j goes to sum j), added by a
+// fixed tree; eight independent chains hide the fp64 add latency, which a
+// single chain pays once per chunk (1600 chunks in a 100 MiB fp32 bucket).
 __device__ void reduce_bucket(const PlanView& v, int64_t b, double* G, int lane) {
   const int K = v.K, P = tri(K);
   const int64_t c0 = v.chunk_prefix[b], c1 = v.chunk_prefix[b + 1];
   for (int p = lane; p < P; p += 32) {
-    double s = 0.0;
+    double t[8] = {0.0, 0.0, 0.0, 0.0, 0.0, 0.0, 0.0, 0.0};
     const double* src = v.partials + c0 * P + p;
-    for (int64_t c = c0; c < c1; ++c, src += P) s += *src;
+    int64_t c = c0;
+    for (; c + 8 <= c1; c += 8, src += 8 * P) {
+#pragma unroll
+      for (int j = 0; j < 8; ++j) t[j] += src[j * P];
+    }
+#pragma unroll
+    for (int j = 0; j < 8; ++j)
+      if (c + j < c1) t[j] += src[j * P];
+    const double s = ((t[0] + t[1]) + (t[2] + t[3])) + ((t[4] + t[5]) + (t[6] + t[7]));
     int i = 0, r = p;
     while (r >= K - i) {
       r -= K - i;
