@@ -1,6 +1,9 @@
 // Host side of the C ABI (include/bkmoo.h): argument checks, the bucket plan,
-// the workspace image and the launch sequence Gram -> solve -> combine on the
-// caller's stream.  Nothing here allocates device memory.
+// the workspace image, the launch sequence Gram -> solve -> combine on the
+// caller's stream (whole plan, a bucket range, or windows of buckets staged
+// from host memory), and the fused persistent launch.  Nothing here
+// allocates device memory (the host path creates two copy streams and a few
+// events per call).
 #include <cuda_runtime.h>
 
 #include <cstring>
@@ -15,7 +18,7 @@ using namespace bkmoo;
 
 namespace {
 
-constexpr int32_t kVersion = 100;  // 0.1.0
+constexpr int32_t kVersion = 200;  // 0.2.0: bucket-range and host-memory entry points
 
 bool offsets_ok(const int64_t* off, int64_t B) {
   if (!off || B < 0 || off[0] != 0) return false;

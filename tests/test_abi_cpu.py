@@ -43,7 +43,7 @@ def test_library_exports_every_declared_symbol():
 
 
 def test_version_and_status_strings():
-    assert bk.bkmoo_version() == 100
+    assert bk.bkmoo_version() == 200
     for code in range(8):
         assert bk.bkmoo_status_string(code) != "unknown status"
     assert bk.bkmoo_status_string(99) == "unknown status"
