@@ -78,6 +78,14 @@ typedef enum { BKMOO_F32 = 0, BKMOO_BF16 = 1 } bkmoo_dtype;
                                           bucket is still in L2 (K <= 8; for
                                           larger K the flag is ignored and
                                           the three-pass path runs)          */
+#define BKMOO_FLAG_TEST_WITHHOLD 0x100u /* testing failure detection, with
+                                          BKMOO_FLAG_FUSED only: the fused
+                                          kernel never publishes bucket 0's
+                                          coefficients, so its bounded waits
+                                          (about 1 s) run out and the call
+                                          ends with BKMOO_ERR_TIMEOUT in the
+                                          workspace status word; the output
+                                          is then undefined                 */
 
 typedef struct {
   int32_t max_iter; /* Frank-Wolfe iterations per bucket (MGDA, CAGrad)     */

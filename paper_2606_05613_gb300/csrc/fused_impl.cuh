@@ -187,7 +187,9 @@ __device__ __noinline__ void fused_solver_cta(const FusedView& f, const SolvePar
       }
       if (lane == 0 && f.out_status) f.out_status[b] = st;
       __syncwarp();
-      if (lane == 0) {
+      // BKMOO_FLAG_TEST_WITHHOLD: bucket 0 is never published, so every
+      // wait on it runs out (the failure-detection test)
+      if (lane == 0 && !(b == 0 && (prm.flags & BKMOO_FLAG_TEST_WITHHOLD))) {
         __threadfence();
         atomicExch(f.ready + b, 1);
       }

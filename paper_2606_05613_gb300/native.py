@@ -31,6 +31,7 @@ BKMOO_F32, BKMOO_BF16 = 0, 1
 BKMOO_FLAG_CLOSED_FORM_K2 = 0x1
 BKMOO_FLAG_POLISH = 0x2
 BKMOO_FLAG_FUSED = 0x4
+BKMOO_FLAG_TEST_WITHHOLD = 0x100
 BKMOO_NOALLOC_SCRATCH_BYTES = 32 << 20
 BKMOO_NOALLOC_MAX_BUCKETS = 4096
 

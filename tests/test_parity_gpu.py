@@ -381,6 +381,33 @@ def test_fused_workspace_mismatch_is_detected():
     assert res.status() == 0
 
 
+def test_fused_bounded_wait_reports_timeout():
+    """Failure detection without a fault: with bucket 0's coefficients never
+    published (a flag that nothing sets), every wait of the persistent kernel
+    ends after its bound, the call reports BKMOO_ERR_TIMEOUT through the
+    workspace status word, and the context stays usable: the next resolve
+    succeeds and matches the oracle."""
+    import time
+    w = _workload(4, "bf16", RAGGED, 150000, seed=23)
+    off = bk.bkmoo_plan(w.param_sizes, w.elem_bytes, w.bucket_bytes)
+    grads = inputs.generate(w, off, DEV)
+    res = bk.Resolver(4, torch.bfloat16, off, DEV)
+    out = torch.empty(int(off[-1]), dtype=torch.bfloat16, device=DEV)
+    p = _fused_params(flags=bk.bkmoo_default_params().flags | bk.BKMOO_FLAG_TEST_WITHHOLD)
+    t0 = time.time()
+    res.resolve(grads, "mgda", out, params=p)
+    assert res.status() == bk.BKMOO_ERR_TIMEOUT
+    assert time.time() - t0 < 30.0
+    B = len(off) - 1
+    beta = torch.empty(B, 4, device=DEV)
+    status = torch.empty(B, dtype=torch.int32, device=DEV)
+    res.resolve(grads, "mgda", out, params=_fused_params(), out_weights=beta, out_status=status)
+    torch.cuda.synchronize()
+    assert res.status() == 0
+    hv = [inputs.host_view(g) for g in grads]
+    _check_against_oracle(w, "mgda", off, hv, out, beta.cpu().numpy(), status.cpu().numpy(), "bf16")
+
+
 @pytest.mark.parametrize("K", [2, 4, 8, 16])
 def test_conflict_statistics(K):
     """Figure 1 statistics from the GPU Gram against the oracle's (cosines to
