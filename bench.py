@@ -47,6 +47,10 @@ def _args():
     ap.add_argument("--path", default="3pass", choices=["fused", "3pass"],
                     help="fused: one persistent launch per step (re-read from L2); "
                          "3pass: Gram, solve and combination launches")
+    ap.add_argument("--hook", action="store_true",
+                    help="time a synthetic training step of a GPT-2-small-shaped transformer "
+                         "with the per-bucket resolve inside the backward pass (BucketMOO) "
+                         "against plain gradient accumulation")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=3)
@@ -290,10 +294,103 @@ def run_reference(a):
     print(json.dumps(line), flush=True)
 
 
+def run_hook(a):
+    """One training step = K languages' forward + backward on their own
+    synthetic token batches.  BucketMOO: gradients land in the bucket layout
+    and each bucket is resolved (MGDA) on a side stream as soon as the last
+    language's backward pass completes it (Algorithm 1); baseline: the same
+    passes accumulating into .grad (the averaged update of plain fine-tuning).
+    Prints one JSON line with both step times."""
+    import numpy as np
+    import torch
+
+    from paper_2606_05613_gb300 import build as nb
+    from paper_2606_05613_gb300 import native as bk
+    from paper_2606_05613_gb300.hook import BucketMOO
+    nb.build()
+    bk.load()
+    dev = torch.device("cuda", 0)
+    torch.manual_seed(0)
+    V, D, L, H, F, T, Bt, K = 50257, 768, 12, 12, 3072, 512, 8, 4
+
+    class Model(torch.nn.Module):
+        def __init__(self):
+            super().__init__()
+            self.emb = torch.nn.Embedding(V, D)
+            self.pos = torch.nn.Embedding(T, D)
+            layer = torch.nn.TransformerEncoderLayer(D, H, F, dropout=0.0, activation="gelu",
+                                                     batch_first=True, norm_first=True)
+            self.body = torch.nn.TransformerEncoder(layer, L, enable_nested_tensor=False)
+            self.norm = torch.nn.LayerNorm(D)
+
+        def forward(self, x):
+            h = self.emb(x) + self.pos.weight[: x.shape[1]]
+            mask = torch.nn.Transformer.generate_square_subsequent_mask(x.shape[1], device=x.device)
+            h = self.norm(self.body(h, mask=mask, is_causal=True))
+            return h @ self.emb.weight.t()          # tied head
+
+    model = Model().to(dev)
+    params = [p for p in model.parameters() if p.requires_grad]
+    n_params = sum(p.numel() for p in params)
+    gen = torch.Generator(device=dev).manual_seed(1)
+    batches = [torch.randint(0, V, (Bt, T + 1), device=dev, generator=gen) for _ in range(K)]
+
+    def loss_of(k):
+        x = batches[k]
+        logits = model(x[:, :-1])
+        return torch.nn.functional.cross_entropy(logits.reshape(-1, V), x[:, 1:].reshape(-1))
+
+    moo = BucketMOO(params, K, 25 << 20, rule=a.rule if a.rule != "mean" else "mgda")
+
+    def step_moo():
+        for k in range(K):
+            moo.begin(k)
+            loss_of(k).backward()
+        moo.finish()
+
+    def step_plain():
+        for p in params:
+            p.grad = None
+        for k in range(K):
+            (loss_of(k) / K).backward()
+
+    def timed(fn):
+        for _ in range(a.warmup):
+            fn()
+        torch.cuda.synchronize(dev)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        for _ in range(a.steps):
+            fn()
+        e1.record()
+        torch.cuda.synchronize(dev)
+        return e0.elapsed_time(e1) / a.steps
+
+    t_plain = timed(step_plain)
+    t_moo = timed(step_moo)
+    moo.remove()
+    print(json.dumps({
+        "metric": "training step with per-bucket MOO resolve inside the backward pass",
+        "unit": "ms", "n_gpus": 1, "steps": a.steps, "warmup": a.warmup, "data": "synthetic",
+        "dtype": "f32", "higher_is_better": False,
+        "config": {"model": "GPT-2-small-shaped transformer (12 x 768, tied 50257 vocab)",
+                   "n_params": n_params, "K": K, "batch_per_language": Bt, "seq_len": T,
+                   "rule": moo.rule, "n_buckets": moo.layout.n_buckets,
+                   "bucket_bytes": 25 << 20},
+        "ms_per_step_bucket_moo": t_moo, "ms_per_step_plain_accumulation": t_plain,
+        "overhead": t_moo / t_plain - 1.0,
+        "bucket_status_counts": {str(k): int(v) for k, v in
+                                 zip(*np.unique(moo.status.cpu().numpy(), return_counts=True))},
+    }), flush=True)
+
+
 def main():
     a = _args()
     if a.impl == "reference":
         run_reference(a)
+        return
+    if a.hook:
+        run_hook(a)
         return
     import numpy as np
     import torch
