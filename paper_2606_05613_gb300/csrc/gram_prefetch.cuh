@@ -40,41 +40,71 @@ __device__ __forceinline__ void cp_async_wait() {
   asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
 }
 
-// find_bucket with, after the hint, a guess that is exact when the buckets
-// from the hint on have the hint's chunk count (one tensor cut into equal
-// buckets): with one CTA per SM a CTA's next chunk lies about 152 chunks on,
-// many small buckets away, and the binary search's dependent loads sit on
-// the path of the copies this kernel issues.  (The other kernels keep the
-// plain search: the guess costs them registers and occupancy.)
-__device__ __forceinline__ int64_t find_bucket_guess(const int64_t* cp, int64_t B, int64_t w,
-                                                     int64_t hint) {
-  if (hint < B && cp[hint] <= w) {
-    const int64_t c0 = cp[hint], c1 = cp[hint + 1];
-    if (w < c1) return hint;
-    const int64_t g = hint + (w - c0) / (c1 > c0 ? c1 - c0 : 1);
-    if (g < B && cp[g] <= w && w < cp[g + 1]) return g;
+// The bucket of a CTA's current chunk with its chunk and element bounds in
+// registers.  A CTA's next chunk lies gridDim.x chunks on, with one CTA per
+// SM often many small buckets away; a plain search then costs several
+// dependent global loads on the path of the copies this kernel issues.
+// seek() guesses the bucket from the current bucket's chunk count (exact
+// when the buckets have equal chunk counts, as one tensor cut into equal
+// buckets does) and loads the guess's four bounds in one round trip; a wrong
+// guess falls back to find_bucket.  (The other kernels keep the plain
+// search: these registers would cost them occupancy.)
+struct BucketTracker {
+  int64_t b, c0, c1, o0, o1;
+  __device__ void load(const PlanView& v, int64_t bb) {
+    b = bb;
+    c0 = v.chunk_prefix[bb];
+    c1 = v.chunk_prefix[bb + 1];
+    o0 = v.offsets[bb];
+    o1 = v.offsets[bb + 1];
   }
-  return find_bucket(cp, B, w, hint);
-}
+  __device__ void init(const PlanView& v) { load(v, v.b_lo < v.n_buckets ? v.b_lo : 0); }
+  __device__ void seek(const PlanView& v, int64_t w) {
+    if (c0 <= w && w < c1) return;
+    if (c0 <= w) {
+      const int64_t g = b + (w - c0) / (c1 - c0);
+      if (g < v.n_buckets) {
+        const int64_t g0 = v.chunk_prefix[g], g1 = v.chunk_prefix[g + 1];
+        const int64_t h0 = v.offsets[g], h1 = v.offsets[g + 1];
+        if (g0 <= w && w < g1) {
+          b = g;
+          c0 = g0;
+          c1 = g1;
+          o0 = h0;
+          o1 = h1;
+          return;
+        }
+      }
+    }
+    load(v, find_bucket(v.chunk_prefix, v.n_buckets, w, b));
+  }
+  // chunk w's element range [s, e) and vector range [vs, vs + nv * EPV)
+  template <int EPV>
+  __device__ void range(const PlanView& v, int64_t w, int64_t* s, int64_t* e, int64_t* vs,
+                        int* nv) const {
+    *s = o0 + (w - c0) * v.chunk_elems;
+    *e = min(*s + v.chunk_elems, o1);
+    int64_t a = (*s + EPV - 1) / EPV * EPV;
+    if (a > *e) a = *e;
+    int64_t z = *e / EPV * EPV;
+    if (z < a) z = a;
+    *vs = a;
+    *nv = (int)((z - a) / EPV);
+  }
+};
 
 // This thread's sequence of 16-byte positions: chunk w = c_lo + blockIdx.x,
 // + gridDim.x, ...; within a chunk the vectors i = t, t + 256, ... < nv.
 template <int EPV>
 struct VecCursor {
-  int64_t w, b, vs;
+  BucketTracker bt;
+  int64_t w, vs;
   int nv, i;
   __device__ void settle(const PlanView& v) {
     while (w < v.c_hi) {
-      b = find_bucket_guess(v.chunk_prefix, v.n_buckets, w, b);
-      const int64_t be = v.offsets[b + 1];
-      const int64_t s = v.offsets[b] + (w - v.chunk_prefix[b]) * v.chunk_elems;
-      const int64_t e = min(s + v.chunk_elems, be);
-      int64_t a = (s + EPV - 1) / EPV * EPV;
-      if (a > e) a = e;
-      int64_t z = e / EPV * EPV;
-      if (z < a) z = a;
-      vs = a;
-      nv = (int)((z - a) / EPV);
+      bt.seek(v, w);
+      int64_t s, e;
+      bt.range<EPV>(v, w, &s, &e, &vs, &nv);
       if (i < nv) return;
       w += gridDim.x;
       i = threadIdx.x;
@@ -82,7 +112,7 @@ struct VecCursor {
   }
   __device__ void begin(const PlanView& v) {
     w = v.c_lo + blockIdx.x;
-    b = v.b_lo;
+    bt.init(v);
     i = threadIdx.x;
     settle(v);
   }
@@ -129,17 +159,14 @@ __global__ void __launch_bounds__(kThreads) gram_prefetch_kernel(const GradPtrs 
   for (int j = 0; j < S - 1; ++j) issue();
 
   int consumed = 0;
-  int64_t b = v.b_lo;
+  BucketTracker ct;
+  ct.init(v);
   for (int64_t w = v.c_lo + blockIdx.x; w < v.c_hi; w += gridDim.x) {
-    b = find_bucket_guess(v.chunk_prefix, v.n_buckets, w, b);
-    const int64_t be = v.offsets[b + 1];
-    const int64_t s0 = v.offsets[b] + (w - v.chunk_prefix[b]) * v.chunk_elems;
-    const int64_t e = min(s0 + v.chunk_elems, be);
-    int64_t vs = (s0 + EPV - 1) / EPV * EPV;
-    if (vs > e) vs = e;
-    int64_t ve = e / EPV * EPV;
-    if (ve < vs) ve = vs;
-    const int nv = (int)((ve - vs) / EPV);
+    ct.seek(v, w);
+    int64_t s0, e, vs;
+    int nv;
+    ct.range<EPV>(v, w, &s0, &e, &vs, &nv);
+    const int64_t ve = vs + (int64_t)nv * EPV;
 
     float acc[P];
 #pragma unroll
