@@ -42,7 +42,8 @@ def _args():
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", default="qwen3-8b",
-                    help="qwen3-8b | llama3.2-1b | gpt2-small | tiny | sweep-K-MiB")
+                    help="qwen3-8b | llama3.2-1b | gpt2-small | tiny | sweep-K-MiB[-<n>M]; "
+                         "append -global for one bucket over every parameter")
     ap.add_argument("--rule", default="mgda", choices=["mgda", "pcgrad", "cagrad", "mean"])
     ap.add_argument("--path", default="3pass", choices=["fused", "3pass"],
                     help="fused: one persistent launch per step (re-read from L2); "
@@ -70,6 +71,12 @@ def workload(name):
         return inputs.tiny()
     if name.startswith("qwen3-8b-") and name.endswith("layers"):
         return inputs.qwen3_8b_layers(int(name[len("qwen3-8b-"):-len("layers")]))
+    if name.endswith("-global"):
+        # the conventional (global) MOO of the paper's Table 2: one bucket
+        # holding every parameter
+        import dataclasses
+        w = workload(name[: -len("-global")])
+        return dataclasses.replace(w, name=w.name + "-global", bucket_bytes=1 << 62)
     if name.startswith("sweep-"):
         # sweep-K-MiB, or sweep-K-MiB-<n>M for a vector of n million elements
         parts = name.split("-")

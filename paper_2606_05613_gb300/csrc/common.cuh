@@ -22,6 +22,12 @@ constexpr int kVecPerThread = 16;          // 16-byte vectors per thread per Gra
 constexpr uint32_t kMagic = 0x4f4d4b42u;   // "BKMO"
 constexpr int kSolveWarpsPerBlock = 4;
 constexpr int kFusedMaxCtas = 2048;        // upper bound of the fused grid
+// A bucket with more than kGroupMinChunks chunks has its chunk partials
+// pre-reduced in groups of kGroupChunks (group_reduce_kernel, solve.cu)
+// before the per-bucket reduction reads them: one warp would otherwise read
+// every partial of a huge bucket (the one-bucket "global" variant) alone.
+constexpr int64_t kGroupChunks = 512;
+constexpr int64_t kGroupMinChunks = 1024;
 
 __host__ __device__ constexpr int tri(int K) { return K * (K + 1) / 2; }
 __host__ __device__ constexpr int elems_per_vec(int dtype) { return dtype == BKMOO_F32 ? 4 : 8; }
@@ -103,6 +109,7 @@ struct PlanView {
   // [b_lo, b_hi) (the whole plan except in the windowed host-memory path).
   int64_t c_lo, c_hi;
   int64_t b_lo, b_hi;
+  int64_t max_chunks;   // most chunks in one bucket of the plan (host-computed)
 };
 
 // Whole-plan window of a view whose n_buckets and n_chunks are set.
@@ -252,5 +259,8 @@ const void* fused_fn_bf16_k7_8(int K, int dtype_out);
 cudaError_t launch_solve(const PlanView& v, const SolveParams& p, float* out_weights,
                          int32_t* out_status, cudaStream_t s);
 cudaError_t launch_gram_finalize(const PlanView& v, double* out_gram, cudaStream_t s);
+// After a Gram pass over the view's window: the group pre-reduction of its
+// large buckets (a no-op when no bucket has more than kGroupMinChunks chunks).
+cudaError_t launch_group_reduce(const PlanView& v, cudaStream_t s);
 
 }  // namespace bkmoo

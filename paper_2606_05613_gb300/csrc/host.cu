@@ -177,6 +177,11 @@ int prepare(const void* const* grads, int32_t K, int32_t dt, const int64_t* offs
   v->plan_hash = plan_hash(K, dt, offsets, B);
   v->K = K;
   v->in_dtype = dt;
+  v->max_chunks = 0;
+  for (int64_t b = 0; b < B; ++b) {
+    const int64_t n = (offsets[b + 1] - offsets[b] + ch - 1) / ch;
+    if (n > v->max_chunks) v->max_chunks = n;
+  }
   full_window(*v);
   std::memset(g, 0, sizeof(*g));
   for (int k = 0; k < K; ++k) g->p[k] = grads[k];
@@ -202,6 +207,7 @@ int launch_gram_pass(const GradPtrs& g, const PlanView& v, cudaStream_t s, bool 
   void* args[] = {&ga, &va};
   if (cudaLaunchKernel(fn, dim3(grid), dim3(kThreads), args, smem, s) != cudaSuccess)
     return BKMOO_ERR_CUDA;
+  if (launch_group_reduce(v, s) != cudaSuccess) return BKMOO_ERR_CUDA;
   return BKMOO_OK;
 }
 

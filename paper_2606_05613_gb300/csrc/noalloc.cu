@@ -162,6 +162,11 @@ extern "C" int bkmoo_gram_noalloc(const void* const* grads, int32_t K, int32_t i
   v.plan_hash = t.hdr.plan_hash;
   v.K = K;
   v.in_dtype = in_dtype;
+  v.max_chunks = 0;
+  for (int64_t b = 0; b < n_buckets; ++b) {
+    const int64_t nb = (offsets[b + 1] - offsets[b] + ch - 1) / ch;
+    if (nb > v.max_chunks) v.max_chunks = nb;
+  }
   full_window(v);
   GradPtrs g;
   std::memset(&g, 0, sizeof g);
@@ -184,6 +189,7 @@ extern "C" int bkmoo_gram_noalloc(const void* const* grads, int32_t K, int32_t i
   void* args[] = {&g, &v};
   if (cudaLaunchKernel(fn, dim3((unsigned)grid), dim3(kThreads), args, smem, s) != cudaSuccess)
     return BKMOO_ERR_CUDA;
+  if (launch_group_reduce(v, s) != cudaSuccess) return BKMOO_ERR_CUDA;
   if (launch_gram_finalize(v, out_gram, s) != cudaSuccess) return BKMOO_ERR_CUDA;
   return BKMOO_OK;
 }

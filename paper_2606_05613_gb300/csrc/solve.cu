@@ -48,7 +48,46 @@ __global__ void __launch_bounds__(32 * kSolveWarpsPerBlock)
   for (int i = lane; i < K * K; i += 32) out_gram[b * K * K + i] = G[i];
 }
 
+// Block (x = group j, y-stride over buckets b): for a bucket of more than
+// kGroupMinChunks chunks, thread p < K(K+1)/2 sums entry p over the chunks
+// [c0 + 512 j, c0 + 512 (j+1)) of the bucket (eight interleaved fp64 sums,
+// fixed tree) and writes the result into the group's first row.  Each
+// (row, entry) is read and written by one thread only.
+__global__ void __launch_bounds__(256) group_reduce_kernel(const PlanView v) {
+  if (!header_ok(v)) return;
+  const int P = tri(v.K);
+  const int p = threadIdx.x;
+  if (p >= P) return;
+  for (int64_t b = v.b_lo + blockIdx.y; b < v.b_hi; b += gridDim.y) {
+    const int64_t cb0 = v.chunk_prefix[b], cb1 = v.chunk_prefix[b + 1];
+    if (cb1 - cb0 <= kGroupMinChunks) continue;
+    const int64_t c0 = cb0 + (int64_t)blockIdx.x * kGroupChunks;
+    if (c0 >= cb1) continue;
+    const int64_t c1 = min(c0 + kGroupChunks, cb1);
+    double t[8] = {0.0, 0.0, 0.0, 0.0, 0.0, 0.0, 0.0, 0.0};
+    const double* src = v.partials + c0 * P + p;
+    int64_t c = c0;
+    for (; c + 8 <= c1; c += 8, src += 8 * P) {
+#pragma unroll
+      for (int j = 0; j < 8; ++j) t[j] += src[j * P];
+    }
+#pragma unroll
+    for (int j = 0; j < 8; ++j)
+      if (c + j < c1) t[j] += src[j * P];
+    v.partials[c0 * P + p] = ((t[0] + t[1]) + (t[2] + t[3])) + ((t[4] + t[5]) + (t[6] + t[7]));
+  }
+}
+
 }  // namespace
+
+cudaError_t launch_group_reduce(const PlanView& v, cudaStream_t s) {
+  if (v.max_chunks <= kGroupMinChunks || v.b_hi <= v.b_lo) return cudaSuccess;
+  const int64_t gx = (v.max_chunks + kGroupChunks - 1) / kGroupChunks;
+  int64_t gy = v.b_hi - v.b_lo;
+  if (gy > 65535) gy = 65535;
+  group_reduce_kernel<<<dim3((unsigned)gx, (unsigned)gy), 256, 0, s>>>(v);
+  return cudaGetLastError();
+}
 
 cudaError_t launch_solve(const PlanView& v, const SolveParams& p, float* out_weights,
                          int32_t* out_status, cudaStream_t s) {

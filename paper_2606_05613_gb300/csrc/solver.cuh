@@ -60,20 +60,29 @@ constexpr double kPivot = 1e-13;   // smallest pivot of a non-singular system
 // interleaved fp64 running sums (chunk c0 + 8m + j goes to sum j), added by a
 // fixed tree; eight independent chains hide the fp64 add latency, which a
 // single chain pays once per chunk (1600 chunks in a 100 MiB fp32 bucket).
+// A bucket of more than kGroupMinChunks chunks was pre-reduced by
+// group_reduce_kernel: its group sums sit in the rows of the first chunk of
+// each group of kGroupChunks, and those rows are what is summed here.
 __device__ void reduce_bucket(const PlanView& v, int64_t b, double* G, int lane) {
   const int K = v.K, P = tri(K);
-  const int64_t c0 = v.chunk_prefix[b], c1 = v.chunk_prefix[b + 1];
+  int64_t c0 = v.chunk_prefix[b], c1 = v.chunk_prefix[b + 1];
+  int64_t stride = 1;  // in chunks
+  if (c1 - c0 > kGroupMinChunks) {
+    stride = kGroupChunks;
+    c1 = c0 + (c1 - c0 + kGroupChunks - 1) / kGroupChunks;  // c0 + number of groups
+  }
+  const int64_t rs = stride * P;  // doubles between the rows summed
   for (int p = lane; p < P; p += 32) {
     double t[8] = {0.0, 0.0, 0.0, 0.0, 0.0, 0.0, 0.0, 0.0};
     const double* src = v.partials + c0 * P + p;
     int64_t c = c0;
-    for (; c + 8 <= c1; c += 8, src += 8 * P) {
+    for (; c + 8 <= c1; c += 8, src += 8 * rs) {
 #pragma unroll
-      for (int j = 0; j < 8; ++j) t[j] += src[j * P];
+      for (int j = 0; j < 8; ++j) t[j] += src[j * rs];
     }
 #pragma unroll
     for (int j = 0; j < 8; ++j)
-      if (c + j < c1) t[j] += src[j * P];
+      if (c + j < c1) t[j] += src[j * rs];
     const double s = ((t[0] + t[1]) + (t[2] + t[3])) + ((t[4] + t[5]) + (t[6] + t[7]));
     int i = 0, r = p;
     while (r >= K - i) {

@@ -307,6 +307,39 @@ def test_global_variant_is_one_bucket(dt):
         _check_against_oracle(w, rule, one, hv, out, beta.cpu().numpy(), status.cpu().numpy(), dt)
 
 
+@pytest.mark.parametrize("dt", ["f32", "bf16"])
+def test_huge_buckets_group_reduction(dt):
+    """Buckets of more than 1024 chunks (their chunk partials are pre-reduced
+    in groups of 512 before the per-bucket sum): Gram and every rule against
+    the oracle, with ragged last groups, a small bucket between two large
+    ones, and bit-identical results run to run."""
+    K = 3
+    ch = 16384 if dt == "f32" else 32768
+    sizes = [1025 * ch + 7, 5000, 2048 * ch + 3]          # 1026, 1 and 2049 chunks
+    w = _workload(K, dt, sizes, 1)
+    off = np.concatenate([[0], np.cumsum(list(reversed(sizes)))]).astype(np.int64)
+    grads = inputs.generate(w, off, DEV)
+    hv = [inputs.host_view(g) for g in grads]
+    B = len(off) - 1
+    res = bk.Resolver(K, _tdt(dt), off, DEV)
+    G = torch.empty(B, K, K, dtype=torch.float64, device=DEV)
+    res.gram(grads, G)
+    G1 = G.cpu().numpy()
+    res.gram(grads, G)
+    np.testing.assert_array_equal(G1, G.cpu().numpy())
+    for b in range(B):
+        ok, err = gram_close(G1[b], orc.gram(hv, int(off[b]), int(off[b + 1] - off[b])))
+        assert ok, (b, err)
+    for rule in ("mgda", "pcgrad", "cagrad"):
+        out = torch.empty(int(off[-1]), dtype=_tdt(dt), device=DEV)
+        beta = torch.empty(B, K, device=DEV)
+        status = torch.empty(B, dtype=torch.int32, device=DEV)
+        res.resolve(grads, rule, out, out_weights=beta, out_status=status)
+        torch.cuda.synchronize()
+        assert res.status() == 0
+        _check_against_oracle(w, rule, off, hv, out, beta.cpu().numpy(), status.cpu().numpy(), dt)
+
+
 # ---------------------------------------------------------------------------
 # fused path (BKMOO_FLAG_FUSED): one persistent launch per resolve
 # ---------------------------------------------------------------------------
