@@ -235,3 +235,23 @@ def test_resolve_buckets_rejects_bad_ranges_without_launch():
     assert call(2, 1) == bk.BKMOO_ERR_INVALID
     assert call(1, 1) == bk.BKMOO_OK            # empty range: nothing queued
     assert call(0, 3, wsb=64) == bk.BKMOO_ERR_WORKSPACE
+
+
+def test_plan_one_bucket_global_variant():
+    """The conventional (global) MOO is the one-bucket plan: a bucket size
+    larger than the model puts every tensor into one bucket."""
+    sizes = inputs.gpt2_small_sizes()
+    off = bk.bkmoo_plan(sizes, 4, 1 << 62)
+    np.testing.assert_array_equal(off, [0, sum(sizes)])
+    np.testing.assert_array_equal(off, orc.plan(sizes, 4, 1 << 62))
+
+
+def test_bench_workload_names():
+    import sys
+    sys.path.insert(0, ROOT)
+    import bench
+    w = bench.workload("qwen3-8b-global")
+    assert w.bucket_bytes == 1 << 62 and w.K == 4 and w.dtype == "bf16"
+    w = bench.workload("sweep-16-1-64M")
+    assert w.K == 16 and w.bucket_bytes == 1 << 20 and sum(w.param_sizes) == 64_000_000
+    assert bench.workload("sweep-2-100").param_sizes == (1_000_000_000,)
