@@ -175,6 +175,18 @@ class ClockSampler:
                 "reasons": reasons, "samples": len(rows)}
 
 
+def launches_per_step(w, off, fused):
+    """Kernels of this library one resolve launches: the fused kernel; or
+    Gram pass, solve and combination, plus the group pre-reduction of the
+    chunk partials when a bucket has more than 1024 chunks."""
+    import numpy as np
+    if fused and w.K <= 8:
+        return 1
+    ch = 16384 if w.dtype == "f32" else 32768
+    longest = int(np.max(np.diff(np.asarray(off, dtype=np.int64))))
+    return 3 + (1 if (longest + ch - 1) // ch > 1024 else 0)
+
+
 def base_config(w, off, rule):
     """The workload description both arms print."""
     return {"workload": w.name, "K": w.K, "grad_dtype": w.dtype, "out_dtype": w.dtype,
@@ -518,7 +530,7 @@ def main():
                           "frac_2k1_of_measured": step_bytes_2k1 / (ms_step * 1e-3) / GB / peak,
                           "frac_k1_of_measured": step_bytes_k1 / (ms_step * 1e-3) / GB / peak,
                           "frac_2k1_of_8tbs": step_bytes_2k1 / (ms_step * 1e-3) / GB / 8000.0},
-        "gpu_launches": (1 if fused else 3) * a.steps,
+        "gpu_launches": launches_per_step(w, off, fused) * a.steps,
         "clocks": clk,
         "bucket_status_counts": {str(k): int((st == k).sum()) for k in sorted(set(st.tolist()))},
         "host_wall_ms_per_step": 1e3 * wall / a.steps,
