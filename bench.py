@@ -38,7 +38,7 @@ GB = 1e9
 def _args():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--steps", type=int, default=50)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", default="qwen3-8b",
@@ -210,46 +210,56 @@ def reduce_over_ranks(ms_step, grad_bytes, device):
     return ms, float(u.item()) / (ms * 1e-3) / GB
 
 
-def cpu_baseline(w, offsets, seconds, n_threads=0, rule="mgda"):
-    """The oracle, as it stands, on a bounded sample of the workload's
-    buckets (host-generated with the same generator), repeated until about
-    `seconds` of wall time; returns (GB/s of gradient bytes, cores, sample)."""
+def cpu_sample(w, offsets, cores):
+    """A bounded sample of the workload for the CPU oracle: one bucket per
+    core, spread over the model, host-generated with the same generator.
+    Returns (K host arrays, sample offsets, the picked bucket indices)."""
+    import numpy as np
     import torch
 
-    from oracle import oracle as orc
     from paper_2606_05613_gb300 import inputs
-    cores = orc.max_threads() if n_threads <= 0 else n_threads
     B = len(offsets) - 1
     n_s = min(B, max(1, cores))
-    # buckets spread over the model, each bucket generated on its own
     picks = sorted(set(int(round(i * (B - 1) / max(1, n_s - 1))) for i in range(n_s)))
-    sub_sizes = [int(offsets[b + 1] - offsets[b]) for b in picks]
     sub_off = [0]
-    for s in sub_sizes:
-        sub_off.append(sub_off[-1] + s)
-    import numpy as np
+    for b in picks:
+        sub_off.append(sub_off[-1] + int(offsets[b + 1] - offsets[b]))
     hv = [np.empty(sub_off[-1], dtype=np.float32 if w.dtype == "f32" else np.uint16)
           for _ in range(w.K)]
-    # generate each picked bucket directly into the sample arrays
+    tdt = torch.float32 if w.dtype == "f32" else torch.bfloat16
     for i, b in enumerate(picks):
         lo, hi = int(offsets[b]), int(offsets[b + 1])
-        tdt = torch.float32 if w.dtype == "f32" else torch.bfloat16
         bufs = [torch.empty(hi - lo, dtype=tdt) for _ in range(w.K)]
         _generate_bucket(w, offsets, b, bufs)
         for k in range(w.K):
             hv[k][sub_off[i]:sub_off[i + 1]] = inputs.host_view(bufs[k])
+    return hv, np.array(sub_off, dtype=np.int64), picks
+
+
+def oracle_pass(hv, sub_off, rule, cores):
+    """One pass of the oracle, as it stands, over the sample; returns seconds."""
+    from oracle import oracle as orc
     t0 = time.perf_counter()
-    passes = 0
+    orc.resolve(hv, sub_off, getattr(orc, rule.upper()), n_threads=cores)
+    return time.perf_counter() - t0
+
+
+def cpu_baseline(w, offsets, seconds, n_threads=0, rule="mgda"):
+    """The oracle on a bounded sample of the workload's buckets, repeated
+    until about `seconds` of wall time; returns (GB/s of gradient bytes,
+    cores, sample description, seconds per pass)."""
+    from oracle import oracle as orc
+    cores = orc.max_threads() if n_threads <= 0 else n_threads
+    hv, sub_off, picks = cpu_sample(w, offsets, cores)
+    dt, passes = 0.0, 0
     while True:
-        orc.resolve(hv, np.array(sub_off, dtype=np.int64), getattr(orc, rule.upper()),
-                    n_threads=cores)
+        dt += oracle_pass(hv, sub_off, rule, cores)
         passes += 1
-        if time.perf_counter() - t0 >= seconds:
+        if dt >= seconds:
             break
-    dt = time.perf_counter() - t0
-    grad_bytes = w.K * sub_off[-1] * w.elem_bytes * passes
+    grad_bytes = w.K * int(sub_off[-1]) * w.elem_bytes * passes
     sample = ("%d of %d buckets (%d elements per language), %d passes, %s"
-              % (len(picks), B, sub_off[-1], passes, rule))
+              % (len(picks), len(offsets) - 1, int(sub_off[-1]), passes, rule))
     return grad_bytes / dt / GB, cores, sample, dt / passes
 
 
@@ -287,17 +297,17 @@ def run_reference(a):
     orc.build()
     w = workload(a.workload)
     off = orc.plan(w.param_sizes, w.elem_bytes, w.bucket_bytes)
-    # each step: one oracle pass over a sample of one bucket per core
-    for _ in range(a.warmup):
-        cpu_baseline(w, off, 0.0, rule=a.rule)
-    vals, times = [], []
+    # each step: one oracle pass over a sample of one bucket per core (the
+    # sample is generated once, outside the timed passes)
     cores = orc.max_threads()
-    sample = ""
-    for _ in range(a.steps):
-        v, cores, sample, t = cpu_baseline(w, off, 0.0, rule=a.rule)
-        vals.append(v)
-        times.append(t)
-    v = sum(vals) / len(vals)
+    hv, sub_off, picks = cpu_sample(w, off, cores)
+    for _ in range(a.warmup):
+        oracle_pass(hv, sub_off, a.rule, cores)
+    times = [oracle_pass(hv, sub_off, a.rule, cores) for _ in range(a.steps)]
+    step_bytes = w.K * int(sub_off[-1]) * w.elem_bytes
+    v = step_bytes * len(times) / sum(times) / GB
+    sample = ("%d of %d buckets (%d elements per language), one pass per step, %s"
+              % (len(picks), len(off) - 1, int(sub_off[-1]), a.rule))
     line = {
         "impl": "reference", "metric": "bucket-MOO resolve GB/s of K-language grads",
         "value": v, "unit": "GB/s", "n_gpus": a.gpus, "steps": a.steps, "warmup": a.warmup,
