@@ -528,6 +528,98 @@ void bko_pcgrad(int32_t K, const double* G, uint64_t seed, uint64_t step,
   if (near_ties) *near_ties = ties;
 }
 
+/*
+ * Every result PCGrad can give when each near-tie test may go either way.
+ * The conflict test <d_t, g_j> < 0 of Eq. 5 / Algorithm 1 is discontinuous:
+ * where |<d_t, g_j>| <= 1e-6 ||d_t|| ||g_j|| (the near-tie bound of
+ * bko_pcgrad) a rounding difference in the Gram can flip it, and both
+ * "project" and "keep" are correct outcomes.  Row t of C (the coefficients of
+ * d_t) depends on no other row, so the alternatives are enumerated per task:
+ * a depth-first walk of t's order that follows both branches at every near
+ * tie (the projection branch only when ||g_j|| > 0), collecting the distinct
+ * final rows.  beta = sum_t row_t, so the results are every sum of one
+ * alternative row per task, enumerated with task 0 varying slowest.
+ * Returns the number of results written to betas (n x K, row-major), or -1
+ * when there are more than cap.  With no near tie the single result is
+ * bko_pcgrad's.
+ */
+#define PCG_ROWS_MAX 64
+static int pcg_rows(int K, const double* Gn, const int32_t* order, int q,
+                    double* row, double* rows, int n, int cap) {
+  for (; q < K - 1; ++q) {
+    int j = order[q];
+    double p = 0.0;
+    for (int m = 0; m < K; ++m) p += row[m] * Gn[m * K + j];
+    double dd = quad_form(K, Gn, row);
+    int tie = fabs(p) <= 1e-6 * sqrt(fabs(dd) * Gn[j * K + j]);
+    int can = Gn[j * K + j] > 0.0;
+    if (tie && can) {
+      double alt[KMAX];
+      memcpy(alt, row, sizeof(double) * K);
+      alt[j] -= p / Gn[j * K + j];
+      n = pcg_rows(K, Gn, order, q + 1, alt, rows, n, cap);
+      if (n < 0) return -1;
+      /* the other branch continues below without the projection */
+    } else if (p < 0.0 && can) {
+      row[j] -= p / Gn[j * K + j];
+    }
+  }
+  for (int i = 0; i < n; ++i) {
+    int same = 1;
+    for (int m = 0; m < K; ++m)
+      if (rows[i * K + m] != row[m]) same = 0;
+    if (same) return n;
+  }
+  if (n >= cap) return -1;
+  memcpy(rows + n * K, row, sizeof(double) * K);
+  return n + 1;
+}
+
+int32_t bko_pcgrad_alternatives(int32_t K, const double* G, uint64_t seed,
+                                uint64_t step, int64_t bucket, int32_t cap,
+                                double* betas) {
+  double Gn[KMAX * KMAX];
+  static const int rows_cap = PCG_ROWS_MAX;
+  double* rows = (double*)malloc(sizeof(double) * KMAX * rows_cap * KMAX);
+  int nrow[KMAX];
+  int32_t order[KMAX];
+  if (!rows) return -1;
+  normalise(K, G, Gn);
+  long total = 1;
+  for (int t = 0; t < K; ++t) {
+    double row[KMAX];
+    for (int m = 0; m < K; ++m) row[m] = (m == t) ? 1.0 : 0.0;
+    bko_pcgrad_order(seed, step, bucket, K, t, order);
+    nrow[t] = pcg_rows(K, Gn, order, 0, row, rows + t * rows_cap * KMAX, 0,
+                       rows_cap);
+    if (nrow[t] < 0) {
+      free(rows);
+      return -1;
+    }
+    total *= nrow[t];
+    if (total > cap) {
+      free(rows);
+      return -1;
+    }
+  }
+  for (long r = 0; r < total; ++r) {
+    int pick[KMAX];
+    long rem = r;
+    for (int t = K - 1; t >= 0; --t) {
+      pick[t] = (int)(rem % nrow[t]);
+      rem /= nrow[t];
+    }
+    double* out = betas + r * K;
+    for (int m = 0; m < K; ++m) {
+      double s = 0.0;
+      for (int t = 0; t < K; ++t) s += rows[t * rows_cap * KMAX + pick[t] * K + m];
+      out[m] = s;
+    }
+  }
+  free(rows);
+  return (int32_t)total;
+}
+
 /* ------------------------------------------------------------------------ */
 /* CAGrad (Eq. 4; bucket form Eq. 7; the CAGrad branch of Algorithm 1).      */
 /* ------------------------------------------------------------------------ */

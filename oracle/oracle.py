@@ -84,6 +84,8 @@ def _load():
         lib.bko_pcgrad_order.argtypes = [u64, u64, i64, i32, i32, vp]
         lib.bko_pcgrad.restype = None
         lib.bko_pcgrad.argtypes = [i32, vp, u64, u64, i64, vp, vp]
+        lib.bko_pcgrad_alternatives.restype = i32
+        lib.bko_pcgrad_alternatives.argtypes = [i32, vp, u64, u64, i64, i32, vp]
         lib.bko_cagrad.restype = None
         lib.bko_cagrad.argtypes = [i32, vp, dbl, vp, vp]
         lib.bko_conflicts.restype = None
@@ -197,6 +199,19 @@ def pcgrad(G, seed: int, step: int, bucket: int):
     ties = np.zeros(1, dtype=np.int32)
     _load().bko_pcgrad(K, _ptr(G), seed, step, bucket, _ptr(b), _ptr(ties))
     return b, int(ties[0])
+
+
+def pcgrad_alternatives(G, seed: int, step: int, bucket: int, cap: int = 256) -> np.ndarray:
+    """Every PCGrad result when each near-tie conflict test may go either way
+    (n x K array of beta; one row, equal to pcgrad()'s, when there is no near
+    tie).  Raises when there are more than `cap` results."""
+    G = _as_G(G)
+    K = G.shape[0]
+    out = np.zeros((cap, K))
+    n = _load().bko_pcgrad_alternatives(K, _ptr(G), seed, step, bucket, cap, _ptr(out))
+    if n < 0:
+        raise ValueError("more than %d PCGrad alternatives" % cap)
+    return out[:n].copy()
 
 
 def cagrad(G, c: float):

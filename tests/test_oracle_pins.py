@@ -210,7 +210,7 @@ def test_mgda_brute_force_grid_k3():
         assert abs(a.sum() - 1) < 1e-12 and (a >= 0).all()
 
 
-@pytest.mark.parametrize("K", [3, 4, 5, 8, 12])
+@pytest.mark.parametrize("K", [3, 4, 5, 8, 12, 16])
 def test_mgda_wolfe_vs_enumeration(K):
     rng = np.random.default_rng(100 + K)
     for trial in range(20):
@@ -419,6 +419,78 @@ def test_pcgrad_no_conflict_is_plain_sum():
         np.testing.assert_array_equal(beta, np.ones(K))
 
 
+def _pcgrad_literal_all(vs, seed, step, bucket):
+    """Algorithm 1's PCGrad branch on materialised fp64 vectors, taking both
+    outcomes of every conflict test that lies within the near-tie bound
+    |<d_t, g_j>| <= 1e-6 ||d_t|| ||g_j||: every direction d it can return."""
+    K = len(vs)
+    g = [v.astype(np.float64) for v in vs]
+
+    def walk(d, order, q):
+        if q == len(order):
+            return [d]
+        j = order[q]
+        p = float(np.dot(d, g[j]))
+        nn = float(np.dot(g[j], g[j]))
+        tie = abs(p) <= 1e-6 * math.sqrt(float(np.dot(d, d)) * nn)
+        if tie and nn > 0:
+            return walk(d - p / nn * g[j], order, q + 1) + walk(d, order, q + 1)
+        if p < 0 and nn > 0:
+            d = d - p / nn * g[j]
+        return walk(d, order, q + 1)
+
+    per_task = [walk(g[t].copy(), orc.pcgrad_order(seed, step, bucket, K, t), 0)
+                for t in range(K)]
+    return [sum(ds) for ds in itertools.product(*per_task)]
+
+
+def test_pcgrad_alternatives_without_ties_is_pcgrad():
+    rng = np.random.default_rng(16)
+    for K in (2, 3, 5, 8, 16):
+        for trial in range(6):
+            G = _gram_np(_rand_vectors(rng, K, 3 * K, corr=rng.uniform(-0.8, 0.8),
+                                       flip_odd=bool(trial % 2)))
+            beta, ties = orc.pcgrad(G, 2, trial, 11)
+            alts = orc.pcgrad_alternatives(G, 2, trial, 11)
+            if ties == 0:
+                assert alts.shape == (1, K)
+                np.testing.assert_array_equal(alts[0], beta)
+
+
+def test_pcgrad_alternatives_match_literal_at_near_ties():
+    """Knife-edge conflicts (a pair whose inner product is a tiny multiple of
+    the norms, of either sign): the set of PCGrad results over both branches
+    of each near tie equals the set of directions that Algorithm 1 on the
+    materialised vectors gives with the tied tests taken either way."""
+    rng = np.random.default_rng(17)
+    seen_multi = 0
+    for K in (2, 3, 4, 6):
+        for trial in range(8):
+            n = 4 * K
+            vs = _rand_vectors(rng, K, n, corr=rng.uniform(-0.6, 0.6), flip_odd=bool(trial % 2))
+            # make (0, 1) a near-orthogonal pair: remove the component of g1
+            # along g0, then add back a tiny multiple (sign by trial)
+            g0, g1 = vs[0], vs[1]
+            g1 = g1 - np.dot(g1, g0) / np.dot(g0, g0) * g0
+            eps = (1e-9 if trial % 4 < 2 else -1e-9) * np.linalg.norm(g1) / np.linalg.norm(g0)
+            vs[1] = g1 + eps * g0
+            G = _gram_np(vs)
+            beta, ties = orc.pcgrad(G, 3, trial, 5)
+            alts = orc.pcgrad_alternatives(G, 3, trial, 5)
+            X = np.stack(vs)
+            got = [a @ X for a in alts]
+            ref = _pcgrad_literal_all(vs, 3, trial, 5)
+            scale = np.abs(X).max() * K
+            for d in ref:                       # every literal outcome is an alternative
+                assert min(np.abs(d - e).max() for e in got) <= 1e-9 * scale
+            for e in got:                       # and every alternative is a literal outcome
+                assert min(np.abs(d - e).max() for d in ref) <= 1e-9 * scale
+            assert any(np.abs(beta - a).max() <= 1e-12 for a in alts)
+            assert (len(alts) > 1) <= (ties > 0)
+            seen_multi += len(alts) > 1
+    assert seen_multi >= 8
+
+
 # ----------------------------------------------------------------------------
 # CAGrad (Eq. 4, Eq. 7, Theorem 3.2)
 # ----------------------------------------------------------------------------
@@ -446,25 +518,65 @@ def test_cagrad_c0_is_mean_and_k1():
     np.testing.assert_allclose(beta, [1.3], atol=1e-15)
 
 
-@pytest.mark.parametrize("K", [2, 3, 4, 6])
+def _cagrad_certificate(vs, c):
+    """Optimality certificate of the oracle's CAGrad answer on materialised
+    vectors (Eq. 4 / Eq. 7): d = beta X is feasible with the constraint
+    active, w lies on the simplex, and the primal value min_k <g_k, d> equals
+    the dual value F(w) (by weak duality min_k <g_k, d> <= F(w') for every
+    feasible d and every w' on the simplex, so equality proves both optimal);
+    plus the bound of Theorem 3.2 (a)."""
+    G = _gram_np(vs)
+    beta, w = orc.cagrad(G, c)
+    X = np.stack(vs)
+    d = beta @ X
+    g0 = X.mean(axis=0)
+    n0 = float(np.linalg.norm(g0))
+    assert (w >= 0).all() and abs(w.sum() - 1) <= 1e-12
+    assert abs(np.linalg.norm(d - g0) - c * n0) <= 1e-9 * n0
+    prim = min(float(np.dot(v, d)) for v in vs)
+    dual = _F(G, w, c)
+    assert abs(prim - dual) <= 1e-9 * np.diag(G).max()
+    assert float(np.dot(g0, d)) >= (1 - c * c) / 2 * n0 * n0 - 1e-9 * n0 * n0
+    return G, w
+
+
+@pytest.mark.parametrize("K", [2, 3, 4, 6, 8, 12, 16])
 def test_cagrad_primal_properties(K):
-    """Constraint active, zero duality gap (min_k <g_k, d> equals the dual
-    value) and the bound of Theorem 3.2 (a), on materialised vectors."""
+    """Constraint active, zero duality gap and Theorem 3.2 (a) on random
+    materialised vectors, aligned or with the shared part flipped on odd
+    languages."""
     rng = np.random.default_rng(20 + K)
     for trial in range(15):
         c = [0.5, 0.2, 0.9][trial % 3]
         vs = _rand_vectors(rng, K, 5 * K, corr=rng.uniform(-0.9, 0.9), flip_odd=bool(trial % 2))
-        G = _gram_np(vs)
-        beta, w = orc.cagrad(G, c)
-        X = np.stack(vs)
-        d = beta @ X
-        g0 = X.mean(axis=0)
-        n0 = float(np.linalg.norm(g0))
-        assert abs(np.linalg.norm(d - g0) - c * n0) <= 1e-9 * n0
-        prim = min(float(np.dot(v, d)) for v in vs)
-        dual = _F(G, w, c)
-        assert abs(prim - dual) <= 1e-9 * np.diag(G).max()
-        assert float(np.dot(g0, d)) >= (1 - c * c) / 2 * n0 * n0 - 1e-9 * n0 * n0
+        _cagrad_certificate(vs, c)
+
+
+@pytest.mark.parametrize("K", [3, 5, 8, 12, 16])
+def test_cagrad_opposed_language_certificate(K):
+    """One language sign-flipped over a strong shared part (<g_k, g0> < 0 for
+    it, the GPU parity workload's conflict case): the same certificate, and
+    the dual minimiser beats random points of the simplex (Dirichlet draws,
+    dense and sparse)."""
+    rng = np.random.default_rng(60 + K)
+    done = 0
+    for trial in range(12):
+        vs = _rand_vectors(rng, K, 6 * K, corr=rng.uniform(0.6, 0.95))
+        k = int(rng.integers(K))
+        vs[k] = -vs[k]
+        g0 = np.stack(vs).mean(axis=0)
+        if np.dot(vs[k], g0) >= 0:      # the flipped language dominates the mean
+            continue
+        done += 1
+        G, w = _cagrad_certificate(vs, 0.5)
+        Fw = _F(G, w, 0.5)
+        for alpha in (1.0, 0.1):
+            W = rng.dirichlet(np.full(K, alpha), size=20000)
+            b = G.sum(axis=1) / K
+            g0n = math.sqrt(G.sum() / K / K)
+            vals = W @ b + 0.5 * g0n * np.sqrt(np.clip(np.einsum("ni,ij,nj->n", W, G, W), 0, None))
+            assert Fw <= vals.min() + 1e-12 * np.diag(G).max()
+    assert done >= 4
 
 
 def test_cagrad_primal_brute_force_low_dimension():
