@@ -137,16 +137,22 @@ int64_t bko_plan(const int64_t* sizes, int32_t n_params, int32_t elem_bytes,
 /* Gram matrix of one bucket (the inner products of Eq. 2, Eq. 6, Eq. 8).    */
 /* ------------------------------------------------------------------------ */
 
-/* G[i*K+j] = sum_{e in [begin, begin+n)} x_i[e] * x_j[e], summed in order. */
+/* G[i*K+j] = sum_{e in [begin, begin+n)} x_i[e] * x_j[e], each entry summed
+ * sequentially in increasing e (one pass over the elements, every entry i <= j
+ * keeping its own running sum). */
 void bko_gram(int32_t K, int32_t dtype, const void* const* x, int64_t begin,
               int64_t n, double* G) {
+  double s[KMAX * KMAX], v[KMAX];
+  for (int32_t i = 0; i < K * K; ++i) s[i] = 0.0;
+  for (int64_t e = begin; e < begin + n; ++e) {
+    for (int32_t i = 0; i < K; ++i) v[i] = load_elem(x[i], dtype, e);
+    for (int32_t i = 0; i < K; ++i)
+      for (int32_t j = i; j < K; ++j) s[i * K + j] += v[i] * v[j];
+  }
   for (int32_t i = 0; i < K; ++i)
     for (int32_t j = i; j < K; ++j) {
-      double s = 0.0;
-      for (int64_t e = begin; e < begin + n; ++e)
-        s += load_elem(x[i], dtype, e) * load_elem(x[j], dtype, e);
-      G[i * K + j] = s;
-      G[j * K + i] = s;
+      G[i * K + j] = s[i * K + j];
+      G[j * K + i] = s[i * K + j];
     }
 }
 
