@@ -200,9 +200,11 @@ int bkmoo_conflicts(const double* gram, int32_t K, int64_t n_buckets, float* out
  * gradients (half as many with fp32); larger problems return
  * BKMOO_ERR_WORKSPACE.
  *
- * The first call on each device (with that device current) looks up the
- * array's device address once (cudaGetSymbolAddress); make that first call
- * before any stream capture.  Every call shares the one array and rewrites
+ * Each call made outside stream capture looks up the array's device address
+ * in the current context (cudaGetSymbolAddress, with the device current);
+ * a call made while its stream is being captured reuses the last address
+ * seen on that device, so make the first call on each device before any
+ * stream capture.  Every call shares the one array and rewrites
  * the parts it reads, so results never depend on an earlier call; but calls
  * whose work overlaps on the GPU (other streams or host threads on the same
  * device) race on it and must be serialised by the caller.
@@ -339,6 +341,24 @@ const char* bkmoo_status_string(int32_t status);
 
 /* Library version, major * 10000 + minor * 100 + patch. */
 int32_t bkmoo_version(void);
+
+/*
+ * bkmoo_selftest_fp64 -- runs, element by element on the device, the fp64
+ * division and square root that the fast per-bucket solvers use for the
+ * CAGrad and PCGrad coefficients (Eq. 4 / Eq. 7, Eq. 5 / Eq. 8): an fp32
+ * seed refined by one Newton-Raphson step with a residual correction
+ * (q = a r, q + (a - b q) r with r = 1/b rounded to fp32; s + (x - s^2) / (2 s)
+ * with s = sqrt(x) rounded to fp32), relative error at most about 2^-46;
+ * arguments outside [1e-30, 1e30] take the correctly rounded operation.
+ * A test entry point, so that its accuracy can be checked against the
+ * correctly rounded fp64 operations.
+ * op 0: out[i] = a[i] / b[i]; op 1: out[i] = sqrt(a[i]) (0 for a[i] <= 0;
+ * b unused, may be NULL).  a, b, out: device fp64 [n].  Asynchronous on
+ * `stream`.  Returns BKMOO_ERR_INVALID for another op, n < 0 or a NULL
+ * array, BKMOO_ERR_CUDA if the launch fails.
+ */
+int bkmoo_selftest_fp64(int32_t op, const double* a, const double* b, double* out, int64_t n,
+                        void* stream);
 
 #ifdef __cplusplus
 }

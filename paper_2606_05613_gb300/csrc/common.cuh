@@ -66,6 +66,38 @@ struct WsLayout {
 
 __host__ __device__ inline size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
 
+// Host-side plan helpers shared by every entry point.
+// Offsets start at 0 and increase strictly (no empty bucket).
+inline bool offsets_ok(const int64_t* off, int64_t B) {
+  if (!off || B < 0 || off[0] != 0) return false;
+  for (int64_t b = 0; b < B; ++b)
+    if (off[b + 1] <= off[b]) return false;
+  return true;
+}
+
+// Gram chunks of a plan: each bucket is cut into chunks of ch elements, the
+// last one short.
+inline int64_t count_chunks(const int64_t* off, int64_t B, int64_t ch) {
+  int64_t n = 0;
+  for (int64_t b = 0; b < B; ++b) n += (off[b + 1] - off[b] + ch - 1) / ch;
+  return n;
+}
+
+// FNV-1a over the 64-bit words that define a plan (K, dtype, B, offsets);
+// kept in the workspace header and checked by every kernel.
+inline uint64_t plan_hash(int32_t K, int32_t dt, const int64_t* off, int64_t B) {
+  uint64_t h = 0xcbf29ce484222325ull;
+  auto mix = [&h](uint64_t x) {
+    h ^= x;
+    h *= 0x100000001b3ull;
+  };
+  mix((uint64_t)K);
+  mix((uint64_t)dt);
+  mix((uint64_t)B);
+  for (int64_t b = 0; b <= B; ++b) mix((uint64_t)off[b]);
+  return h;
+}
+
 __host__ __device__ inline WsLayout ws_layout(int K, int64_t B, int64_t n_chunks) {
   WsLayout L;
   size_t at = sizeof(WsHeader);
@@ -259,6 +291,10 @@ const void* fused_fn_bf16_k7_8(int K, int dtype_out);
 cudaError_t launch_solve(const PlanView& v, const SolveParams& p, float* out_weights,
                          int32_t* out_status, cudaStream_t s);
 cudaError_t launch_gram_finalize(const PlanView& v, double* out_gram, cudaStream_t s);
+// The fp64 division / square-root helpers of the fast solvers, element-wise
+// (self-test of their accuracy against the correctly rounded operations).
+cudaError_t launch_selftest_fp64(int op, const double* a, const double* b, double* out, int64_t n,
+                                 cudaStream_t s);
 // After a Gram pass over the view's window: the group pre-reduction of its
 // large buckets (a no-op when no bucket has more than kGroupMinChunks chunks).
 cudaError_t launch_group_reduce(const PlanView& v, cudaStream_t s);

@@ -20,33 +20,6 @@ namespace {
 
 constexpr int32_t kVersion = 200;  // 0.2.0: bucket-range and host-memory entry points
 
-bool offsets_ok(const int64_t* off, int64_t B) {
-  if (!off || B < 0 || off[0] != 0) return false;
-  for (int64_t b = 0; b < B; ++b)
-    if (off[b + 1] <= off[b]) return false;
-  return true;
-}
-
-int64_t count_chunks(const int64_t* off, int64_t B, int64_t ch) {
-  int64_t n = 0;
-  for (int64_t b = 0; b < B; ++b) n += (off[b + 1] - off[b] + ch - 1) / ch;
-  return n;
-}
-
-// FNV-1a over the 64-bit words that define a plan.
-uint64_t plan_hash(int32_t K, int32_t dt, const int64_t* off, int64_t B) {
-  uint64_t h = 0xcbf29ce484222325ull;
-  auto mix = [&h](uint64_t x) {
-    h ^= x;
-    h *= 0x100000001b3ull;
-  };
-  mix((uint64_t)K);
-  mix((uint64_t)dt);
-  mix((uint64_t)B);
-  for (int64_t b = 0; b <= B; ++b) mix((uint64_t)off[b]);
-  return h;
-}
-
 bool dtype_ok(int32_t dt) { return dt == BKMOO_F32 || dt == BKMOO_BF16; }
 int elem_bytes(int32_t dt) { return dt == BKMOO_F32 ? 4 : 2; }
 bool aligned(const void* p, uintptr_t a) { return ((uintptr_t)p & (a - 1)) == 0; }
@@ -644,5 +617,14 @@ const char* bkmoo_status_string(int32_t status) {
 }
 
 int32_t bkmoo_version(void) { return kVersion; }
+
+int bkmoo_selftest_fp64(int32_t op, const double* a, const double* b, double* out, int64_t n,
+                        void* stream) {
+  if ((op != 0 && op != 1) || n < 0 || (n > 0 && (!a || !out || (op == 0 && !b))))
+    return BKMOO_ERR_INVALID;
+  return launch_selftest_fp64(op, a, b, out, n, static_cast<cudaStream_t>(stream)) == cudaSuccess
+             ? BKMOO_OK
+             : BKMOO_ERR_CUDA;
+}
 
 }  // extern "C"

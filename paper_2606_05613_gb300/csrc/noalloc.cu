@@ -12,9 +12,11 @@
 // process exits.  It calls no cudaMalloc, cudaFree or other allocating routine.
 //
 // Host code never touches g_scratch by name: in host code the name is only a
-// stand-in, not a device address.  The first call on each device (with that
-// device current) looks the address up with cudaGetSymbolAddress and caches
-// it; that first call should come before any stream capture.
+// stand-in, not a device address.  Each call made outside stream capture
+// looks the address up in the current context with cudaGetSymbolAddress
+// (with that device current) and passes it to the kernels; a call made
+// while its stream is being captured reuses the last address seen on that
+// device, so the first call on each device should come before any capture.
 //
 // All calls share the one array and it keeps whatever the last call left
 // there.  Every call rewrites the header (including its status word, which
@@ -64,32 +66,31 @@ __global__ void noalloc_table_kernel(const TableSlice t, unsigned char* scratch,
 std::mutex g_addr_mu;
 void* g_addr[kMaxDevices] = {};
 
-// Device address of g_scratch on the current device (looked up once).
-int scratch_address(unsigned char** out) {
+// Device address of g_scratch in the current context.  Outside stream
+// capture it is looked up on every call (cudaGetSymbolAddress allocates
+// nothing and is cheap once the module is loaded), so a context rebuilt
+// after cudaDeviceReset, or another context made current on the same
+// device, gets its own address; the last address seen on each device is
+// kept for calls made while `s` is being captured, when the runtime call is
+// avoided.  The first call on a device must therefore come before any
+// capture.
+int scratch_address(cudaStream_t s, unsigned char** out) {
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices)
     return BKMOO_ERR_CUDA;
+  cudaStreamCaptureStatus cap = cudaStreamCaptureStatusNone;
+  const bool capturing =
+      cudaStreamIsCapturing(s, &cap) != cudaSuccess || cap != cudaStreamCaptureStatusNone;
+  if (capturing) (void)cudaGetLastError();   // an implicit-capture error is not sticky
   std::lock_guard<std::mutex> lk(g_addr_mu);
-  if (!g_addr[dev]) {
+  if (!capturing) {
     void* p = nullptr;
     if (cudaGetSymbolAddress(&p, g_scratch) != cudaSuccess || !p) return BKMOO_ERR_CUDA;
     g_addr[dev] = p;
   }
+  if (!g_addr[dev]) return BKMOO_ERR_CUDA;   // first call on this device during capture
   *out = static_cast<unsigned char*>(g_addr[dev]);
   return BKMOO_OK;
-}
-
-uint64_t noalloc_plan_hash(int32_t K, int32_t dt, const int64_t* off, int64_t B) {
-  uint64_t h = 0xcbf29ce484222325ull;
-  auto mix = [&h](uint64_t x) {
-    h ^= x;
-    h *= 0x100000001b3ull;
-  };
-  mix((uint64_t)K);
-  mix((uint64_t)dt);
-  mix((uint64_t)B);
-  for (int64_t b = 0; b <= B; ++b) mix((uint64_t)off[b]);
-  return h;
 }
 
 }  // namespace
@@ -101,24 +102,21 @@ extern "C" int bkmoo_gram_noalloc(const void* const* grads, int32_t K, int32_t i
                                   const int64_t* offsets, int64_t n_buckets, double* out_gram,
                                   void* stream) {
   if (K < 1 || K > kMaxK || (in_dtype != BKMOO_F32 && in_dtype != BKMOO_BF16) || !grads ||
-      !offsets || n_buckets < 0 || offsets[0] != 0 || (n_buckets > 0 && !out_gram))
+      !offsets_ok(offsets, n_buckets) || (n_buckets > 0 && !out_gram))
     return BKMOO_ERR_INVALID;
-  for (int64_t b = 0; b < n_buckets; ++b)
-    if (offsets[b + 1] <= offsets[b]) return BKMOO_ERR_INVALID;
   for (int k = 0; k < K; ++k)
     if (!grads[k] || ((uintptr_t)grads[k] & 15u)) return BKMOO_ERR_INVALID;
   const int64_t ch = chunk_elems(in_dtype);
-  int64_t nch = 0;
-  for (int64_t b = 0; b < n_buckets; ++b) nch += (offsets[b + 1] - offsets[b] + ch - 1) / ch;
+  const int64_t nch = count_chunks(offsets, n_buckets, ch);
   const WsLayout L = ws_layout(K, n_buckets, nch);
   if (n_buckets > kNoallocMaxBuckets || L.total > kNoallocScratchBytes)
     return BKMOO_ERR_WORKSPACE;  // larger than the static scratch
   if (n_buckets == 0) return BKMOO_OK;
 
-  unsigned char* scratch = nullptr;
-  int r = scratch_address(&scratch);
-  if (r != BKMOO_OK) return r;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
+  unsigned char* scratch = nullptr;
+  int r = scratch_address(s, &scratch);
+  if (r != BKMOO_OK) return r;
 
   // Bucket table and header, slice by slice through kernel parameters.
   TableSlice t;
@@ -131,7 +129,7 @@ extern "C" int bkmoo_gram_noalloc(const void* const* grads, int32_t K, int32_t i
   t.hdr.n_elems = offsets[n_buckets];
   t.hdr.n_chunks = nch;
   t.hdr.chunk_elems = ch;
-  t.hdr.plan_hash = noalloc_plan_hash(K, in_dtype, offsets, n_buckets);
+  t.hdr.plan_hash = plan_hash(K, in_dtype, offsets, n_buckets);
   int64_t prefix = 0;
   for (int64_t first = 0; first < n_buckets; first += kSlice) {
     const int32_t count = (int32_t)((n_buckets - first) < kSlice ? (n_buckets - first) : kSlice);

@@ -78,7 +78,25 @@ __global__ void __launch_bounds__(256) group_reduce_kernel(const PlanView v) {
   }
 }
 
+// Element i of the fp64 division / square-root helpers of the fast solvers
+// (op 0: a[i] / b[i] by div_nr, op 1: sqrt(a[i]) by sqrt_nr); grid-stride.
+__global__ void selftest_fp64_kernel(int op, const double* a, const double* b, double* out,
+                                     int64_t n) {
+  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n;
+       i += (int64_t)gridDim.x * blockDim.x)
+    out[i] = op == 0 ? div_nr(a[i], b[i]) : sqrt_nr(a[i]);
+}
+
 }  // namespace
+
+cudaError_t launch_selftest_fp64(int op, const double* a, const double* b, double* out, int64_t n,
+                                 cudaStream_t s) {
+  if (n <= 0) return cudaSuccess;
+  int64_t grid = (n + 255) / 256;
+  if (grid > 4096) grid = 4096;
+  selftest_fp64_kernel<<<(unsigned)grid, 256, 0, s>>>(op, a, b, out, n);
+  return cudaGetLastError();
+}
 
 cudaError_t launch_group_reduce(const PlanView& v, cudaStream_t s) {
   if (v.max_chunks <= kGroupMinChunks || v.b_hi <= v.b_lo) return cudaSuccess;

@@ -584,12 +584,19 @@ __device__ int solve_cagrad(int K, const double* G, const SolveParams& p, double
 
 constexpr int kEnumMaxK = 5;
 
-// a / b and sqrt(x) in fp64: an fp32 seed and one Newton-Raphson step
-// (relative error about 2^-46).  Arguments outside the fp32 range take the
-// exact fp64 operation.
+// a / b and sqrt(x) in fp64 by Newton-Raphson from an fp32 seed: for the
+// quotient r = 1/b rounded to fp32, q = a r, then one step with the residual
+// correction q + (a - b q) r; for the root s = sqrt(x) rounded to fp32, then
+// s + (x - s^2) / (2 s) with 1 / (2 s) from the fp32 reciprocal.  The seed
+// carries a relative error of about 2^-23 (two fp32 roundings), which the
+// step squares: at most about 2^-46 (tested against the correctly rounded
+// operations).  Operands where the seed or the intermediate products could
+// leave the fp32 / fp64 normal range (|b| or x outside (1e-30, 1e30), a
+// nonzero |a| outside (1e-270, 1e270)) take the correctly rounded fp64
+// operation instead.
 __device__ __forceinline__ double div_nr(double a, double b) {
-  const double ab = fabs(b);
-  if (!(ab > 1e-30 && ab < 1e30)) return a / b;
+  const double ab = fabs(b), aa = fabs(a);
+  if (!(ab > 1e-30 && ab < 1e30 && aa < 1e270 && (aa > 1e-270 || a == 0.0))) return a / b;
   const double r = (double)__frcp_rn((float)b);
   const double q = a * r;
   return fma(fma(-b, q, a), r, q);

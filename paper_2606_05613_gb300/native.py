@@ -103,6 +103,8 @@ def load():
         lib.bkmoo_status_string.argtypes = [i32]
         lib.bkmoo_version.restype = i32
         lib.bkmoo_version.argtypes = []
+        lib.bkmoo_selftest_fp64.restype = ctypes.c_int
+        lib.bkmoo_selftest_fp64.argtypes = [i32, vp, vp, vp, i64, vp]
         _lib = lib
         return lib
 
@@ -287,6 +289,14 @@ def bkmoo_status_string(code: int) -> str:
 
 def bkmoo_version() -> int:
     return int(load().bkmoo_version())
+
+
+def bkmoo_selftest_fp64(op: int, a, b, out, stream=None):
+    """The solvers' fp64 division (op 0, out = a / b) or square root (op 1,
+    out = sqrt(a)) element-wise on the device (fp64 CUDA tensors)."""
+    _check(load().bkmoo_selftest_fp64(op, a.data_ptr(), b.data_ptr() if b is not None else None,
+                                      out.data_ptr(), int(out.numel()),
+                                      _stream_handle(stream, out.device)), "bkmoo_selftest_fp64")
 
 
 class Resolver:

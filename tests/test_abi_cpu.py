@@ -255,3 +255,62 @@ def test_bench_workload_names():
     w = bench.workload("sweep-16-1-64M")
     assert w.K == 16 and w.bucket_bytes == 1 << 20 and sum(w.param_sizes) == 64_000_000
     assert bench.workload("sweep-2-100").param_sizes == (1_000_000_000,)
+
+
+def _aligned_dummies(n):
+    """n distinct 16-byte-aligned host addresses (never dereferenced: every
+    call below must be rejected before any launch, and on a machine without
+    a GPU a launch would fail with a CUDA error rather than read memory)."""
+    buf = np.zeros(64 * (n + 1), dtype=np.uint8)
+    base = (buf.ctypes.data + 15) & ~15
+    return buf, [base + 64 * i for i in range(n)]
+
+
+def test_gram_noalloc_rejects_bad_arguments_without_launch():
+    lib = bk.load()
+    keep, ptrs_l = _aligned_dummies(17)
+    out = ctypes.c_void_p(ptrs_l[16])
+
+    def call(K, dt, offs, grads=None, out_gram=out, n_buckets=None):
+        ptrs = (ctypes.c_void_p * max(K, 1))(*(grads or ptrs_l[:max(K, 1)]))
+        offs = np.ascontiguousarray(offs, dtype=np.int64)
+        nb_ = len(offs) - 1 if n_buckets is None else n_buckets
+        return lib.bkmoo_gram_noalloc(ptrs, K, dt, offs.ctypes.data, nb_, out_gram, None)
+
+    ok_off = [0, 1000, 2500]
+    # sizes beyond the static scratch: too many buckets, too many elements
+    too_many = np.arange(0, bk.BKMOO_NOALLOC_MAX_BUCKETS + 2, dtype=np.int64)
+    assert call(16, bk.BKMOO_F32, too_many) == bk.BKMOO_ERR_WORKSPACE
+    assert call(16, bk.BKMOO_F32, [0, 10**10]) == bk.BKMOO_ERR_WORKSPACE
+    assert call(4, bk.BKMOO_BF16, [0, 10**11]) == bk.BKMOO_ERR_WORKSPACE
+    # invalid arguments
+    assert call(0, bk.BKMOO_F32, ok_off) == bk.BKMOO_ERR_INVALID
+    assert call(17, bk.BKMOO_F32, ok_off) == bk.BKMOO_ERR_INVALID
+    assert call(4, 7, ok_off) == bk.BKMOO_ERR_INVALID
+    assert call(4, bk.BKMOO_F32, [0, 1000, 1000]) == bk.BKMOO_ERR_INVALID
+    assert call(4, bk.BKMOO_F32, [0, 1000, 900]) == bk.BKMOO_ERR_INVALID
+    assert call(4, bk.BKMOO_F32, [5, 1000, 2500]) == bk.BKMOO_ERR_INVALID
+    assert call(4, bk.BKMOO_F32, ok_off, n_buckets=-1) == bk.BKMOO_ERR_INVALID
+    assert call(4, bk.BKMOO_F32, ok_off, out_gram=None) == bk.BKMOO_ERR_INVALID
+    misaligned = list(ptrs_l[:4])
+    misaligned[2] += 4
+    assert call(4, bk.BKMOO_F32, ok_off, grads=misaligned) == bk.BKMOO_ERR_INVALID
+    nulls = list(ptrs_l[:4])
+    nulls[1] = None
+    assert call(4, bk.BKMOO_F32, ok_off, grads=nulls) == bk.BKMOO_ERR_INVALID
+    assert lib.bkmoo_gram_noalloc(None, 4, bk.BKMOO_F32, np.array(ok_off).ctypes.data, 2, out,
+                                  None) == bk.BKMOO_ERR_INVALID
+    # no bucket: nothing to do, nothing launched
+    assert call(4, bk.BKMOO_F32, [0]) == bk.BKMOO_OK
+    del keep
+
+
+def test_selftest_fp64_rejects_bad_arguments_without_launch():
+    lib = bk.load()
+    keep, p = _aligned_dummies(3)
+    assert lib.bkmoo_selftest_fp64(2, p[0], p[1], p[2], 4, None) == bk.BKMOO_ERR_INVALID
+    assert lib.bkmoo_selftest_fp64(0, p[0], None, p[2], 4, None) == bk.BKMOO_ERR_INVALID
+    assert lib.bkmoo_selftest_fp64(1, None, None, p[2], 4, None) == bk.BKMOO_ERR_INVALID
+    assert lib.bkmoo_selftest_fp64(1, p[0], None, p[2], -1, None) == bk.BKMOO_ERR_INVALID
+    assert lib.bkmoo_selftest_fp64(1, p[0], None, p[2], 0, None) == bk.BKMOO_OK
+    del keep

@@ -9,7 +9,7 @@ from oracle import oracle as orc
 from paper_2606_05613_gb300 import build as nb
 from paper_2606_05613_gb300 import inputs
 from paper_2606_05613_gb300 import native as bk
-from tests.parity_util import BETA_ATOL, beta_unique, d_check, gram_close, widen
+from tests.parity_util import Run, check_window, gram_close, oracle_window
 
 pytestmark = pytest.mark.gpu
 
@@ -60,29 +60,15 @@ def _run(w, rule, out_dt, params=None, inplace=False):
 
 def _check_against_oracle(w, rule, off, hv, out, beta, status, out_dt, seed=0, step=0,
                           mgda_mode=orc.MGDA_EXACT, max_iter=256):
-    ref = orc.resolve(hv, off, ORC_RULE[rule], seed=seed, step=step, cagrad_c=0.5,
-                      mgda_mode=mgda_mode, max_iter=max_iter, want_gram=True)
-    d = out.float().cpu().numpy().astype(np.float64) if out.dtype == torch.bfloat16 else \
-        out.cpu().numpy().astype(np.float64)
+    """Every bucket against the oracle (PCGrad near ties: either branch)."""
     B = len(off) - 1
-    worst = 0.0
-    for b in range(B):
-        lo, hi = int(off[b]), int(off[b + 1])
-        G = ref["gram"][b]
-        gn = np.array([np.linalg.norm(widen(h[lo:hi])) for h in hv])
-        skip_beta = False
-        if rule == "pcgrad":
-            _, ties = orc.pcgrad(G, seed, step, b)
-            if ties:
-                continue
-        elif rule in ("mgda", "cagrad") and not beta_unique(G):
-            skip_beta = True
-        assert status[b] in (0, bk.BKMOO_ERR_NOT_CONVERGED), (b, status[b])
-        if not skip_beta:
-            assert np.abs(beta[b] - ref["beta"][b]).max() <= BETA_ATOL, (b, beta[b], ref["beta"][b])
-        ok, e = d_check(d[lo:hi], ref["d"][lo:hi], ref["beta"][b], gn, out_dt)
-        worst = max(worst, e)
-        assert ok, (rule, out_dt, b, e)
+    run = Run(w.name, np.asarray(off, dtype=np.int64), rule, out, beta, status, out_dt,
+              seed=seed, step=step, mgda_mode=mgda_mode, max_iter=max_iter)
+    if B == 0:
+        return 0.0
+    ref = oracle_window(hv, run.off, 0, B, run)
+    worst = check_window(hv, 0, B, ref, run)
+    assert run.checked == B
     return worst
 
 
