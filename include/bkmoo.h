@@ -77,7 +77,14 @@ typedef enum { BKMOO_F32 = 0, BKMOO_BF16 = 1 } bkmoo_dtype;
                                           bucket after bucket while the
                                           bucket is still in L2 (K <= 8; for
                                           larger K the flag is ignored and
-                                          the three-pass path runs)          */
+                                          the three-pass path runs).  On a
+                                          GB300 it measured slower than the
+                                          three-pass default everywhere: the
+                                          per-bucket solve and hand-offs
+                                          take longer than L2 can hold the
+                                          data streamed meanwhile.  Results
+                                          agree with the three-pass path to
+                                          rounding, not bit for bit.         */
 #define BKMOO_FLAG_TEST_WITHHOLD 0x100u /* testing failure detection, with
                                           BKMOO_FLAG_FUSED only: the fused
                                           kernel never publishes bucket 0's

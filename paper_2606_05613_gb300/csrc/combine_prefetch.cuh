@@ -17,8 +17,13 @@ namespace bkmoo {
 #endif
 constexpr int kCombinePrefetchStages = BKMOO_COMBINE_PREFETCH_STAGES;
 
+// Stages per thread: 4 for K <= 8; 3 above (K = 16: 192 KB of slots, one
+// CTA per SM with 128 KB of copies in flight).
+__host__ __device__ constexpr int combine_prefetch_stages(int K) {
+  return K <= 8 ? kCombinePrefetchStages : 3;
+}
 __host__ __device__ constexpr int combine_prefetch_smem_bytes(int K) {
-  return kCombinePrefetchStages * K * kThreads * 16;
+  return combine_prefetch_stages(K) * K * kThreads * 16;
 }
 
 template <int K, int DTI, int DTO>
@@ -26,7 +31,7 @@ __global__ void __launch_bounds__(kThreads)
     combine_prefetch_kernel(const GradPtrs g, const PlanView v, void* out) {
   constexpr int EPV = elems_per_vec(DTI);
   constexpr int IB = 16 / EPV;
-  constexpr int S = kCombinePrefetchStages;
+  constexpr int S = combine_prefetch_stages(K);
   extern __shared__ __align__(16) unsigned char cpf_smem[];
   uint4* slots = reinterpret_cast<uint4*>(cpf_smem);
   auto slot = [&](int s, int k) -> uint4* { return slots + ((s * K + k) * kThreads + threadIdx.x); };

@@ -22,6 +22,21 @@ constexpr int kVecPerThread = 16;          // 16-byte vectors per thread per Gra
 constexpr uint32_t kMagic = 0x4f4d4b42u;   // "BKMO"
 constexpr int kSolveWarpsPerBlock = 4;
 constexpr int kFusedMaxCtas = 2048;        // upper bound of the fused grid
+// Fused kernel: 11 streaming warps and one solver warp per CTA (12 warps:
+// registers are allocated to warps in groups of four, so 9 warps would cost
+// as many registers as 12); each group of CTAs keeps the CTA partials of its
+// last kFusedRing buckets in a ring.
+constexpr int kFusedStreamWarps = 11;
+constexpr int kFusedThreads = 32 * (kFusedStreamWarps + 1);
+constexpr int kFusedRing = 4;
+// cp.async stages per streaming lane of the fused kernel: about 14 K-vector
+// sets in flight per lane (~80 KB per SM with 11 streaming warps).
+__host__ __device__ constexpr int fused_stages(int K) {
+  return K <= 1 ? 12 : K == 2 ? 8 : K == 3 ? 6 : K == 4 ? 5 : K <= 6 ? 4 : 3;
+}
+__host__ __device__ constexpr int fused_smem_bytes(int K) {
+  return fused_stages(K) * K * 16 * 32 * kFusedStreamWarps;
+}
 // A bucket with more than kGroupMinChunks chunks has its chunk partials
 // pre-reduced in groups of kGroupChunks (group_reduce_kernel, solve.cu)
 // before the per-bucket reduction reads them: one warp would otherwise read
@@ -58,9 +73,10 @@ struct WsLayout {
   size_t beta;           // float [B][K]    coefficients of the last resolve
   size_t total;          // end of the regions above
   // fused path only (bkmoo_resolve with BKMOO_FLAG_FUSED):
-  size_t arrive;         // int32 [B]  streaming CTAs done with bucket b's Gram
-  size_t ready;          // int32 [B]  1 once beta of bucket b is written
-  size_t ring;           // double [2][kFusedMaxCtas][P] per-CTA partials
+  size_t arrive;         // int32 [B]      CTAs of bucket b's group done with its Gram
+  size_t ready;          // int32 [B + 1]  1 once beta of bucket b is written;
+                         //                [B] counts the buckets published
+  size_t ring;           // double [kFusedRing][2 kFusedMaxCtas][P] CTA partials
   size_t total_fused;
 };
 
@@ -113,9 +129,9 @@ __host__ __device__ inline WsLayout ws_layout(int K, int64_t B, int64_t n_chunks
   L.arrive = at;
   at = align256(at + sizeof(int32_t) * (size_t)B);
   L.ready = at;
-  at = align256(at + sizeof(int32_t) * (size_t)B);
+  at = align256(at + sizeof(int32_t) * (size_t)(B + 1));
   L.ring = at;
-  at = align256(at + sizeof(double) * 2 * (size_t)kFusedMaxCtas * (size_t)tri(K));
+  at = align256(at + sizeof(double) * kFusedRing * 2 * (size_t)kFusedMaxCtas * (size_t)tri(K));
   L.total_fused = at;
   return L;
 }
@@ -152,17 +168,18 @@ __host__ __device__ inline void full_window(PlanView& v) {
   v.b_hi = v.n_buckets;
 }
 
-// The fused path's view: the plan plus the synchronisation arrays.
+// The fused path's view: the plan plus the synchronisation arrays.  CTA c
+// belongs to group c % n_groups; bucket b is resolved by group b % n_groups.
 struct FusedView {
   PlanView v;
   int32_t* arrive;
   int32_t* ready;
-  double* ring;
+  double* ring;          // [n_groups][kFusedRing][group_ctas][P]
   float* out_weights;
   int32_t* out_status;
-  int32_t n_stream;      // streaming CTAs; CTA n_stream is the solver
-  int32_t lookahead;     // how far (in 1/1024 of a piece) the Gram of bucket
-                         // b+1 may lead the combination of bucket b
+  int32_t n_groups;
+  int32_t group_ctas;    // rows of a ring slot: CTAs of the largest group
+  int32_t lookahead;     // buckets a warp's Gram may run ahead of its combination
 };
 
 struct SolveParams {
@@ -266,13 +283,14 @@ int gram_prefetch_smem(int K);
 int gram_prefetch_min_k();
 
 // Combine kernels with a per-thread shared-memory prefetch (same signature,
-// combine_prefetch_smem(K) bytes of dynamic shared memory), K <= 8;
-// combine_prefetch.cu.  Measured 2-6.5 % faster than combine_kernel for
-// K = 2..8 (GB300); combine_kernel serves K >= 9.
+// combine_prefetch_smem(K) bytes of dynamic shared memory), every K;
+// combine_prefetch.cu, combine_prefetch_k9_16.cu.  Measured faster than
+// combine_kernel on GB300 (K = 2..8: 2-6.5 %).
 #ifndef BKMOO_COMBINE_PREFETCH
 #define BKMOO_COMBINE_PREFETCH 1
 #endif
 const void* combine_prefetch_fn(int K, int dti, int dto);
+const void* combine_prefetch_fn_k9_16(int K, int dti, int dto);
 int combine_prefetch_smem(int K);
 
 // Combine kernels, signature (GradPtrs, PlanView, void* out); combine_*.cu.

@@ -1,48 +1,71 @@
-// Fused resolve: one persistent, co-resident grid resolves bucket after
-// bucket (Algorithm 1's inner loop over buckets) so that a bucket's
-// gradients are read from HBM once, by the Gram pass, and read again by the
-// combination while they are still in L2.
+// Fused resolve: one persistent, co-resident grid runs Gram -> solve ->
+// combination bucket by bucket (Algorithm 1 resolves each bucket as soon as
+// it is full), so that a bucket's gradients come from HBM once, for the Gram
+// pass, and are read again by the combination while they are still in L2.
 //
-// Roles.  CTAs 0 .. n_stream-1 stream; CTA n_stream solves.
-//  streamer i works on two buckets at once, in small steps (2 vectors per
-//  thread per step), so that HBM reads of the next bucket overlap the solve
-//  and the L2-served combination of the previous one:
-//    Gram of its slice of bucket gb (slice i of n_stream equal, 16-byte-
-//      aligned pieces), loads marked L2 evict_last so that the bucket stays
-//      in L2; the slice's triangle (fp32 per thread over at most 16 vectors,
-//      fixed warp-shuffle tree, fp64 across warps and sub-slices) goes to the
-//      ring of partials, then arrive[gb] += 1 (release).  gb runs at most one
-//      bucket ahead of cb.
-//    combination of its slice of bucket cb once ready[cb] is seen (acquire),
-//      loads marked evict_first (each line is read for the last time),
-//      stores evict_first.  It only blocks (bounded) on ready[cb] when no
-//      Gram step is left to overlap.
-//  solver: for each bucket b, wait until arrive[b] == n_stream (bounded),
-//    reduce the n_stream partials in a fixed order (fp64), solve the rule
-//    (solver.cuh), write beta_b, out_weights, out_status, then ready[b] = 1
-//    (release).
-// A streamer writes the partials of bucket b+2 only after it has seen
-// ready[b], i.e. after the solver has read bucket b's, so two ring slots of
-// partials suffice.  No wait closes a cycle: a streamer blocks on ready[cb]
-// only after arriving for cb and cb+1, and the solver waits only for
-// arrivals.  Every wait gives up after about a second,
-// records BKMOO_ERR_TIMEOUT in the workspace status word and ends the kernel;
-// any recorded error makes every other wait end at once.
+// Why groups.  Between the Gram read of a byte and its re-read, HBM keeps
+// streaming other data; the re-read hits L2 only if everything read in
+// between still fits.  That interval is the bucket's own streaming time plus
+// the latency of its solve and hand-offs, so the grid is split into
+// n_groups groups of CTAs: group g resolves buckets g, g + n_groups, ... one
+// after the other, each bucket spread over the group's CTAs, and the host
+// chooses n_groups so that (lookahead + 1) buckets per group fit the L2
+// budget.  Many small buckets are then in flight at once, each handled by a
+// few dozen CTAs, and every group streams its next bucket(s) while its
+// current one is being solved.
+//
+// CTA layout.  Warps 0..10 stream, warp 11 solves.
+//  A streaming warp owns piece (c_local * 11 + warp) of every bucket of its
+//  group (the bucket's 16-byte vectors cut into group_size * 11 equal
+//  pieces; the unaligned head and tail elements go to the first and last
+//  piece) and walks a fixed schedule of segments: Gram(0) .. Gram(L-1),
+//  then Gram(j + L), Comb(j) for j = 0, 1, ... (L = lookahead).  Each lane
+//  keeps S stages of its next items (the K 16-byte vectors of one position)
+//  in flight with cp.async into its own shared-memory slots, across segment
+//  boundaries: a combination's inputs are prefetched before its beta is
+//  known, since beta is only needed to consume them.
+//    Gram segment: fp32 sums per lane over at most 16 items, fixed butterfly
+//      into fp64 lane-owned entries; at the end the warp stores them in
+//      shared memory, and the last of the 11 warps to finish adds them in a
+//      fixed order, writes the CTA's partial to the group's ring slot and
+//      arrives on arrive[b] (after a fence).  The CTA whose arrival
+//      completes the bucket queues b for its own solver warp.
+//    Comb segment: wait (bounded) for ready[b] (acquire), read beta, then
+//      d = sum_k beta_k g_k over the piece, positions taken from the end of
+//      the piece backwards (the lines read last are reused first).
+//  The solver warp takes queued buckets: it sums the group's CTA partials
+//  in a fixed order (fp64), solves the rule (solver.cuh), writes beta,
+//  out_weights and out_status, fences and sets ready[b]; ready[B] counts the
+//  buckets published.  It leaves when the CTA's streaming warps are done.
+//
+// Ring slots: bucket j of a group uses slot j % kFusedRing.  A warp writes
+// bucket j's partial only while j <= (its next combination) + lookahead, so
+// bucket j - kFusedRing (< j - lookahead - 1) was combined, hence solved,
+// hence its partials were read: kFusedRing > lookahead + 1 suffices.
+//
+// Waits.  Streaming warps wait only for ready flags, the solver warp only
+// for its queue; neither wait closes a cycle (a bucket is queued once all
+// its Gram pieces arrived, and Gram work never waits for a combination).
+// Every wait ends after about a second without progress, records
+// BKMOO_ERR_TIMEOUT in the workspace status word and leaves the kernel; any
+// recorded error ends every other wait at once.
 //
 // The grid must be co-resident (cooperative launch).  Results are
-// deterministic for a given grid size; the chunking differs from the
-// three-pass path, so the two agree to rounding, not bit for bit.
+// deterministic for a given grid and group count; the pieces differ from
+// the three-pass path's chunks, so the two agree to rounding, not bit for
+// bit.
 #pragma once
 
 #include <cuda_bf16.h>
 
 #include "combine_impl.cuh"
-#include "gram_impl.cuh"
+#include "gram_prefetch.cuh"
 #include "solver.cuh"
 
 namespace bkmoo {
 
-constexpr uint64_t kFusedWaitNs = 1000000000ull;  // deadline of one wait: 1 s
+constexpr uint64_t kFusedWaitNs = 1000000000ull;  // a wait gives up after 1 s
+constexpr int kFusedQueue = 16;                    // solver queue entries per CTA
 
 // L2 eviction-priority policies (createpolicy) and 16-byte loads carrying them.
 __device__ __forceinline__ uint64_t policy_evict_last() {
@@ -75,8 +98,8 @@ __device__ __forceinline__ int ld_acquire(const int32_t* p) {
   asm volatile("ld.acquire.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
   return v;
 }
-// A poll that does not order later loads (so it can be issued before a
-// streaming step and read after it); pair a positive poll with fence_acquire.
+// A poll that does not order later loads (issued before a streaming step and
+// read after it); pair a positive poll with fence_acquire.
 __device__ __forceinline__ int ld_relaxed(const int32_t* p) {
   int v;
   asm volatile("ld.relaxed.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(p));
@@ -109,345 +132,413 @@ __device__ __forceinline__ bool fused_wait(const int32_t* p, int target, WsHeade
   return false;
 }
 
-// Slice [lo, hi) of bucket b for streamer i.
+// Piece q of W of bucket b: vectors [vlo, vhi) (in vector units from the
+// bucket's first aligned element vs), plus the bucket's unaligned head
+// [bo, vs) for q == 0 and tail [ve, be) for q == W - 1.
+struct Piece {
+  int64_t bo, be, vs, ve;  // bucket bounds and its aligned vector span (elements)
+  int64_t vlo, vhi;        // this piece's vectors
+};
+
 template <int EPV>
-__device__ __forceinline__ void fused_slice(const PlanView& v, int64_t b, int i, int n,
-                                            int64_t* lo, int64_t* hi) {
-  const int64_t bo = v.offsets[b], be = v.offsets[b + 1];
-  int64_t S = (be - bo + n - 1) / n;
-  S = (S + EPV - 1) / EPV * EPV;
-  int64_t a = bo + (int64_t)i * S;
-  if (a > be) a = be;
-  int64_t z = a + S;
-  if (z > be) z = be;
-  *lo = a;
-  *hi = z;
+__device__ __forceinline__ Piece fused_piece(const PlanView& v, int64_t b, int q, int W) {
+  Piece p;
+  p.bo = v.offsets[b];
+  p.be = v.offsets[b + 1];
+  p.vs = (p.bo + EPV - 1) / EPV * EPV;
+  if (p.vs > p.be) p.vs = p.be;
+  p.ve = p.be / EPV * EPV;
+  if (p.ve < p.vs) p.ve = p.vs;
+  const int64_t nv = (p.ve - p.vs) / EPV;
+  p.vlo = nv * q / W;
+  p.vhi = nv * (q + 1) / W;
+  return p;
+}
+
+// Fixed-order sum of the M CTA partials (rows of P doubles) of one bucket
+// into the symmetric G (shared).  For P <= 16 the rows are split into
+// S = 32 / P stripes (lane l: entry l % P, rows l / P, l / P + S, ...) and the
+// stripe sums are then added in stripe order; for P > 16 lane l owns entries
+// l and l + 32 over all rows.  Each lane adds its rows in increasing order,
+// loading them eight at a time so that the L2 round trips (the rows were
+// written by other CTAs) overlap instead of following one another.
+template <int P, int STRIDE>
+__device__ __forceinline__ double fused_rows_sum(const double* rows, int c0, int M, int p) {
+  double t = 0.0;
+  for (int c = c0; c < M; c += 8 * STRIDE) {
+    double x[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i)
+      x[i] = c + i * STRIDE < M ? __ldcg(rows + (size_t)(c + i * STRIDE) * P + p) : 0.0;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) t += x[i];
+  }
+  return t;
 }
 
 template <int K>
-__device__ __noinline__ void fused_solver_cta(const FusedView& f, const SolveParams& prm) {
+__device__ __forceinline__ void fused_reduce(const double* rows, int M, double* G, int lane) {
   constexpr int P = tri(K);
-  constexpr int STRIPES = kThreads / P > 0 ? kThreads / P : 1;
+  auto put = [&](int p, double t) {
+    int i = 0, r = p;
+    while (r >= K - i) {
+      r -= K - i;
+      ++i;
+    }
+    G[i * K + i + r] = t;
+    G[(i + r) * K + i] = t;
+  };
+  if constexpr (P <= 16) {
+    constexpr int S = 32 / P;
+    const double part = lane < S * P ? fused_rows_sum<P, S>(rows, lane / P, M, lane % P) : 0.0;
+    double tot = 0.0;
+#pragma unroll
+    for (int s = 0; s < S; ++s) tot += __shfl_sync(0xffffffffu, part, s * P + (lane % P));
+    if (lane < P) put(lane, tot);
+  } else {
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+      const int p = lane + 32 * h;
+      if (p < P) put(p, fused_rows_sum<P, 1>(rows, 0, M, p));
+    }
+  }
+}
+
+// The solver warp of a CTA: takes the buckets its CTA completed from the
+// shared-memory queue, reduces, solves and publishes them.
+template <int K>
+__device__ __noinline__ void fused_solver_warp(const FusedView& f, const SolveParams& prm,
+                                               volatile int* queue, volatile int* done_warps) {
+  constexpr int P = tri(K);
   __shared__ double G[K * K];
   __shared__ float Gf[K * K];
-  __shared__ double part[kThreads];
   __shared__ double beta_sh[K];
-  __shared__ int go;
   const PlanView& v = f.v;
-  const int n = f.n_stream;
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  for (int64_t b = 0; b < v.n_buckets; ++b) {
-    if (threadIdx.x == 0) go = fused_wait(f.arrive + b, n, v.hdr) ? 1 : 0;
-    __syncthreads();
-    if (!go) return;
-    // fixed-order reduction of the n CTA partials: thread t sums entry t % P
-    // over stripe t / P of the CTAs with four interleaved accumulators, then
-    // thread e adds its STRIPES stripe sums in order
-    const double* ring = f.ring + (size_t)(b & 1) * kFusedMaxCtas * P;
-    if ((int)threadIdx.x < STRIPES * P) {
-      const int e = threadIdx.x % P, st = threadIdx.x / P;
-      const int c0 = (int)((int64_t)n * st / STRIPES), c1 = (int)((int64_t)n * (st + 1) / STRIPES);
-      double t0 = 0.0, t1 = 0.0, t2 = 0.0, t3 = 0.0;
-      int c = c0;
-      for (; c + 3 < c1; c += 4) {
-        t0 += __ldcg(ring + (size_t)c * P + e);
-        t1 += __ldcg(ring + (size_t)(c + 1) * P + e);
-        t2 += __ldcg(ring + (size_t)(c + 2) * P + e);
-        t3 += __ldcg(ring + (size_t)(c + 3) * P + e);
-      }
-      for (; c < c1; ++c) t0 += __ldcg(ring + (size_t)c * P + e);
-      part[threadIdx.x] = (t0 + t1) + (t2 + t3);
-    }
-    __syncthreads();
-    if ((int)threadIdx.x < P) {
-      double t0 = 0.0, t1 = 0.0;
-      int st = 0;
-      for (; st + 1 < STRIPES; st += 2) {
-        t0 += part[st * P + threadIdx.x];
-        t1 += part[(st + 1) * P + threadIdx.x];
-      }
-      if (st < STRIPES) t0 += part[st * P + threadIdx.x];
-      const double t = t0 + t1;
-      int i = 0, r = threadIdx.x;
-      while (r >= K - i) {
-        r -= K - i;
-        ++i;
-      }
-      G[i * K + i + r] = t;
-      G[(i + r) * K + i] = t;
-    }
-    __syncthreads();
-    if (warp == 0) {
+  const int lane = threadIdx.x & 31;
+  const int64_t B = v.n_buckets;
+  int head = 0;
+  uint64_t t0 = global_ns();
+  int seen = -1;
+  for (unsigned it = 0;; ++it) {
+    const int b32 = queue[head % kFusedQueue];
+    __syncwarp();
+    if (b32 >= 0) {
+      const int64_t b = b32;
+      if (lane == 0) queue[head % kFusedQueue] = -1;
+      ++head;
+      __threadfence();
+      const int64_t grp = b % f.n_groups, j = b / f.n_groups;
+      const int M = (int)((gridDim.x - grp + f.n_groups - 1) / f.n_groups);
+      const double* rows =
+          f.ring + ((size_t)grp * kFusedRing + (size_t)(j % kFusedRing)) * f.group_ctas * P;
+      fused_reduce<K>(rows, M, G, lane);
+      __syncwarp();
       const int st = solver::solve_bucket_warp<K>(K, G, Gf, prm, b, beta_sh, lane);
       if (lane < K) {
         const float fb = (float)beta_sh[lane];
         v.beta[b * K + lane] = fb;
         if (f.out_weights) f.out_weights[b * K + lane] = fb;
-        __threadfence();
       }
       if (lane == 0 && f.out_status) f.out_status[b] = st;
+      __threadfence();
       __syncwarp();
       // BKMOO_FLAG_TEST_WITHHOLD: bucket 0 is never published, so every
       // wait on it runs out (the failure-detection test)
       if (lane == 0 && !(b == 0 && (prm.flags & BKMOO_FLAG_TEST_WITHHOLD))) {
-        __threadfence();
         atomicExch(f.ready + b, 1);
+        atomicAdd(f.ready + B, 1);
+      }
+      __syncwarp();
+      t0 = global_ns();
+      continue;
+    }
+    if ((it & 15u) == 15u) {
+      if (*done_warps == kFusedStreamWarps) return;
+      if (*(volatile int32_t*)&v.hdr->status != 0) return;
+      const int pub = ld_relaxed(f.ready + B);
+      const uint64_t now = global_ns();
+      if (pub != seen) {
+        seen = pub;
+        t0 = now;
+      } else if (now - t0 > kFusedWaitNs) {
+        if (lane == 0) record_error(v.hdr, BKMOO_ERR_TIMEOUT);
+        return;
       }
     }
-    __syncthreads();
+    __nanosleep(32);
   }
 }
 
-// Resident CTAs per SM the register budget is capped for: the streaming
-// loops need up to 128 (K <= 4) and 255 (K > 4) registers per thread; the
-// solver code shares the kernel and spills instead of lowering occupancy.
-template <int K>
-struct FusedMinBlocks {
-  static constexpr int value = K <= 4 ? 2 : 1;
+// A warp's schedule over the J buckets of its group with look-ahead L:
+// Gram(0) .. Gram(L-1), then for j = 0 .. J-1: Gram(j + L) (when
+// j + L < J) and Comb(j).  seg_at(s) gives segment s's (comb, j).
+struct FusedSched {
+  int64_t J;
+  int L;
+  __device__ int64_t prologue() const { return J < L ? J : L; }
+  __device__ int64_t pairs() const { return J > L ? J - L : 0; }
+  __device__ int64_t total() const { return prologue() + J + pairs(); }
+  __device__ void seg_at(int64_t s, bool* comb, int64_t* j) const {
+    const int64_t p0 = prologue(), np = pairs();
+    if (s < p0) {
+      *comb = false;
+      *j = s;
+      return;
+    }
+    const int64_t t = s - p0;
+    if (t < 2 * np) {
+      *comb = (t & 1) != 0;
+      *j = *comb ? t / 2 : t / 2 + L;
+      return;
+    }
+    *comb = true;
+    *j = np + (t - 2 * np);
+  }
 };
 
-// Piece of bucket b streamed by warp w of CTA cta: the CTA's slice cut in
-// kWarps equal, 16-byte-aligned pieces.
-template <int EPV>
-__device__ __forceinline__ void warp_piece(const PlanView& v, int64_t b, int cta, int n, int w,
-                                           int64_t* lo, int64_t* hi) {
-  int64_t a, z;
-  fused_slice<EPV>(v, b, cta, n, &a, &z);
-  int64_t ps = (z - a + kWarps - 1) / kWarps;
-  ps = (ps + EPV - 1) / EPV * EPV;
-  int64_t l = a + (int64_t)w * ps;
-  if (l > z) l = z;
-  int64_t h = l + ps;
-  if (h > z) h = z;
-  *lo = l;
-  *hi = h;
-}
+// Per-lane producer: walks the same segments as the consumer and copies
+// the K vectors of its next item into stage (issued % S) with cp.async;
+// every call commits one group (empty once the schedule is exhausted).
+// Items of a segment: n = ceil(piece vectors / 32) per lane (warp-uniform);
+// item i is vector lo + lane + 32 i of a Gram piece, hi - 1 - (lane + 32 i)
+// of a combination piece (read backwards), valid when inside [lo, hi).
+template <int K, int DT>
+struct FusedProducer {
+  FusedSched sch;
+  int64_t seg, vs, lo, hi, item, n_items;
+  bool comb;
+  int grp, ng, q, W, lane;
+  __device__ void open(const PlanView& v) {
+    while (seg < sch.total()) {
+      int64_t j;
+      sch.seg_at(seg, &comb, &j);
+      const Piece pc = fused_piece<elems_per_vec(DT)>(v, grp + j * ng, q, W);
+      vs = pc.vs;
+      lo = pc.vlo;
+      hi = pc.vhi;
+      n_items = (hi - lo + 31) / 32;
+      item = 0;
+      if (n_items > 0) return;
+      ++seg;
+    }
+  }
+  template <typename Slot>
+  __device__ void issue(const PlanView& v, const GradPtrs& g, Slot slot, int stage) {
+    constexpr int EPV = elems_per_vec(DT);
+    constexpr int IB = 16 / EPV;
+    if (seg < sch.total()) {
+      const int64_t idx = comb ? hi - 1 - (lane + 32 * item) : lo + lane + 32 * item;
+      if (idx >= lo && idx < hi) {
+        const int64_t off = (vs + idx * EPV) * IB;
+#pragma unroll
+        for (int k = 0; k < K; ++k) cp_async16(slot(stage, k), static_cast<const char*>(g.p[k]) + off);
+      }
+      if (++item == n_items) {
+        ++seg;
+        open(v);
+      }
+    }
+    cp_async_commit();
+  }
+};
 
 template <int K, int DT, int DTO>
-__global__ void __launch_bounds__(kThreads, FusedMinBlocks<K>::value)
+__global__ void __launch_bounds__(kFusedThreads, 1)
     fused_resolve_kernel(const GradPtrs g, const FusedView f, const SolveParams prm, void* out) {
   constexpr int P = tri(K);
   constexpr int NP = (P + 31) / 32;       // fp64 accumulators per lane
   constexpr int EPV = elems_per_vec(DT);
-  constexpr int IB = 16 / EPV;
-  constexpr int STEP = K <= 2 ? 4 : 2;    // vectors per lane per Gram / combination step
-  __shared__ double part_sm[2][kWarps][P];
-  __shared__ int cnt_sm[2];
+  constexpr int S = fused_stages(K);
+  __shared__ double part_sm[kFusedRing][kFusedStreamWarps][P];
+  __shared__ int cnt_sm[kFusedRing];
+  __shared__ int queue_sm[kFusedQueue];
+  __shared__ int q_tail, done_warps;
+  extern __shared__ __align__(16) unsigned char fused_smem[];
   const PlanView& v = f.v;
   if (!header_ok(v)) {
-    if (blockIdx.x == 0 && threadIdx.x == 0) record_error(v.hdr, BKMOO_ERR_WORKSPACE);
-    if ((int)blockIdx.x == f.n_stream && f.out_status)
-      for (int64_t b = threadIdx.x; b < v.n_buckets; b += kThreads)
-        f.out_status[b] = BKMOO_ERR_WORKSPACE;
+    if (blockIdx.x == 0) {
+      if (threadIdx.x == 0) record_error(v.hdr, BKMOO_ERR_WORKSPACE);
+      if (f.out_status)
+        for (int64_t b = threadIdx.x; b < v.n_buckets; b += blockDim.x)
+          f.out_status[b] = BKMOO_ERR_WORKSPACE;
+    }
     return;
   }
-  if ((int)blockIdx.x == f.n_stream) {
-    fused_solver_cta<K>(f, prm);
-    return;
+  if (threadIdx.x < kFusedRing) cnt_sm[threadIdx.x] = 0;
+  if (threadIdx.x < kFusedQueue) queue_sm[threadIdx.x] = -1;
+  if (threadIdx.x == 0) {
+    q_tail = 0;
+    done_warps = 0;
   }
-  if (threadIdx.x < 2) cnt_sm[threadIdx.x] = 0;
   __syncthreads();   // the only CTA-wide barrier; every warp runs on its own below
 
-  const int cta = blockIdx.x, n = f.n_stream;
   const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
-  const int64_t B = v.n_buckets;
-  const uint64_t keep = policy_evict_last(), last_use = policy_evict_first();
+  if (wid == kFusedStreamWarps) {
+    fused_solver_warp<K>(f, prm, queue_sm, &done_warps);
+    return;
+  }
 
-  int64_t gb = 0, g_vs = 0, g_nv = 0, g_next = 0;
-  int g_pend = 0;
-  bool g_open = false;
+  // this lane's stage slots: [S][K] 16-byte vectors
+  uint4* my_slots = reinterpret_cast<uint4*>(fused_smem) + (size_t)threadIdx.x * S * K;
+  auto slot = [&](int st, int k) -> uint4* { return my_slots + st * K + k; };
+
+  const int ng = f.n_groups;
+  const int cta = blockIdx.x, grp = cta % ng, c_loc = cta / ng;
+  const int M = (int)((gridDim.x - grp + ng - 1) / ng);
+  const int W = M * kFusedStreamWarps, q = c_loc * kFusedStreamWarps + wid;
+  const int64_t B = v.n_buckets;
+  const FusedSched sch{grp < B ? (B - grp + ng - 1) / ng : 0, f.lookahead};
+
+  FusedProducer<K, DT> pr;
+  pr.sch = sch;
+  pr.seg = 0;
+  pr.grp = grp;
+  pr.ng = ng;
+  pr.q = q;
+  pr.W = W;
+  pr.lane = lane;
+  pr.open(v);
+  int issued = 0;
+#pragma unroll 1
+  for (int j = 0; j < S - 1; ++j) pr.issue(v, g, slot, issued++ % S);
+  int consumed = 0;
+
   float acc[P];
 #pragma unroll
   for (int p = 0; p < P; ++p) acc[p] = 0.0f;
   double acc64[NP];
 #pragma unroll
   for (int i = 0; i < NP; ++i) acc64[i] = 0.0;
-
-  int64_t cb = 0, c_vs = 0, c_nv = 0, c_next = 0;
-  bool c_open = false;
-  float beta[K];
+  auto flush = [&]() {
+    // fixed butterfly over the warp; lane p % 32 keeps entry p in fp64
 #pragma unroll
-  for (int k = 0; k < K; ++k) beta[k] = 0.0f;
-
-  while (cb < B) {
-    // poll for beta of bucket cb now; read the answer after the Gram step
-    const bool want = !c_open && cb < gb;
-    int flag = 0;
-    if (want && lane == 0) flag = ld_relaxed(f.ready + cb);
-
-    // ---- one Gram step of bucket gb: at most one bucket ahead of cb, and
-    // when ahead, at most `lookahead` of a piece ahead of the combination
-    // of cb, so that both buckets' unconsumed lines fit in L2
-    bool gram_ok = gb < B && gb <= cb + 1;
-    if (gram_ok && gb == cb + 1 && g_open) {
-      const int64_t lead = (g_nv * f.lookahead) >> 10;
-      const int64_t follow = c_open ? (c_next * g_nv) / (c_nv > 0 ? c_nv : 1) : 0;
-      gram_ok = g_next < follow + lead;
+    for (int p = 0; p < P; ++p) {
+      float x = acc[p];
+      x += __shfl_xor_sync(0xffffffffu, x, 16);
+      x += __shfl_xor_sync(0xffffffffu, x, 8);
+      x += __shfl_xor_sync(0xffffffffu, x, 4);
+      x += __shfl_xor_sync(0xffffffffu, x, 2);
+      x += __shfl_xor_sync(0xffffffffu, x, 1);
+      if ((p & 31) == lane) acc64[p >> 5] += (double)x;
+      acc[p] = 0.0f;
     }
-    if (gram_ok) {
-      if (!g_open) {
-        int64_t lo, hi;
-        warp_piece<EPV>(v, gb, cta, n, wid, &lo, &hi);
-        g_vs = (lo + EPV - 1) / EPV * EPV;
-        if (g_vs > hi) g_vs = hi;
-        int64_t ve = hi / EPV * EPV;
-        if (ve < g_vs) ve = g_vs;
-        g_nv = (ve - g_vs) / EPV;
-        const int nh = (int)(g_vs - lo), nt = (int)(hi - ve);
-        if (lane < nh + nt) {
-          const int64_t idx = lane < nh ? lo + lane : ve + (lane - nh);
-          gram_accumulate_scalar<K, DT>(acc, g, idx);
-        }
-        g_next = 0;
-        g_pend = 0;
-        g_open = true;
+  };
+
+  bool failed = false;
+  const int64_t total = sch.total();
+  for (int64_t seg = 0; seg < total && !failed; ++seg) {
+    bool comb;
+    int64_t j;
+    sch.seg_at(seg, &comb, &j);
+    const int64_t b = grp + j * ng;
+    const Piece pc = fused_piece<EPV>(v, b, q, W);
+    const int64_t n_items = (pc.vhi - pc.vlo + 31) / 32;
+    if (!comb) {
+      // ---- Gram of this warp's piece of bucket b
+      const int nh = q == 0 ? (int)(pc.vs - pc.bo) : 0;
+      const int nt = q == W - 1 ? (int)(pc.be - pc.ve) : 0;
+      if (lane < nh + nt) {
+        const int64_t idx = lane < nh ? pc.bo + lane : pc.ve + (lane - nh);
+        gram_accumulate_scalar<K, DT>(acc, g, idx);
       }
-      uint4 r[STEP][K];
+      for (int64_t i = 0; i < n_items; ++i) {
+        pr.issue(v, g, slot, issued++ % S);
+        cp_async_wait<S - 1>();
+        const int st = consumed++ % S;
+        if (pc.vlo + lane + 32 * i < pc.vhi) {
+          uint4 r[K];
 #pragma unroll
-      for (int j = 0; j < STEP; ++j) {
-        const int64_t idx = g_next + lane + 32 * j;
-        if (idx < g_nv) {
-#pragma unroll
-          for (int k = 0; k < K; ++k)
-            r[j][k] = ld16_policy_nc(static_cast<const char*>(g.p[k]) + (g_vs + idx * EPV) * IB, keep);
+          for (int k = 0; k < K; ++k) r[k] = *slot(st, k);
+          gram_accumulate<K, DT>(acc, r);
         }
+        if ((i & (kVecPerThread - 1)) == kVecPerThread - 1) flush();
       }
+      flush();
+      // the CTA's warp partials, added in a fixed order by the last warp to
+      // finish, which writes the CTA partial and arrives
+      const int rs = (int)(j % kFusedRing);
 #pragma unroll
-      for (int j = 0; j < STEP; ++j)
-        if (g_next + lane + 32 * j < g_nv) gram_accumulate<K, DT>(acc, r[j]);
-      g_next += 32 * STEP;
-      g_pend += STEP;
-      const bool done = g_next >= g_nv;
-      if (done || g_pend >= kVecPerThread) {
-        // fixed butterfly over the warp; lane p % 32 keeps entry p in fp64
-#pragma unroll
-        for (int p = 0; p < P; ++p) {
-          float x = acc[p];
-          x += __shfl_xor_sync(0xffffffffu, x, 16);
-          x += __shfl_xor_sync(0xffffffffu, x, 8);
-          x += __shfl_xor_sync(0xffffffffu, x, 4);
-          x += __shfl_xor_sync(0xffffffffu, x, 2);
-          x += __shfl_xor_sync(0xffffffffu, x, 1);
-          if ((p & 31) == lane) acc64[p >> 5] += (double)x;
-          acc[p] = 0.0f;
-        }
-        g_pend = 0;
-      }
-      if (done) {
-        // combine the CTA's 8 warp partials in a fixed order; the last warp
-        // to finish publishes the CTA's partial and arrives
-        const int slot = (int)(gb & 1);
-#pragma unroll
-        for (int i = 0; i < NP; ++i)
-          if (lane + 32 * i < P) part_sm[slot][wid][lane + 32 * i] = acc64[i];
+      for (int i = 0; i < NP; ++i)
+        if (lane + 32 * i < P) part_sm[rs][wid][lane + 32 * i] = acc64[i];
+      __threadfence_block();
+      __syncwarp();
+      int last = 0;
+      if (lane == 0) last = (atomicAdd(&cnt_sm[rs], 1) == kFusedStreamWarps - 1) ? 1 : 0;
+      last = __shfl_sync(0xffffffffu, last, 0);
+      if (last) {
         __threadfence_block();
-        __syncwarp();
-        int last = 0;
-        if (lane == 0) last = (atomicAdd(&cnt_sm[slot], 1) == kWarps - 1) ? 1 : 0;
-        last = __shfl_sync(0xffffffffu, last, 0);
-        if (last) {
-          __threadfence_block();
-          double* ring = f.ring + (size_t)slot * kFusedMaxCtas * P + (size_t)cta * P;
+        double* row = f.ring + (((size_t)grp * kFusedRing + rs) * f.group_ctas + c_loc) * P;
 #pragma unroll
-          for (int i = 0; i < NP; ++i) {
-            const int p = lane + 32 * i;
-            if (p < P) {
-              double t = 0.0;
+        for (int i = 0; i < NP; ++i) {
+          const int p = lane + 32 * i;
+          if (p < P) {
+            double t = 0.0;
 #pragma unroll
-              for (int w = 0; w < kWarps; ++w) t += ((volatile double*)part_sm[slot][w])[p];
-              ring[p] = t;
-            }
-          }
-          __threadfence();
-          __syncwarp();
-          if (lane == 0) {
-            cnt_sm[slot] = 0;
-            __threadfence();
-            atomicAdd(f.arrive + gb, 1);
+            for (int w = 0; w < kFusedStreamWarps; ++w) t += ((volatile double*)part_sm[rs][w])[p];
+            __stcg(row + p, t);
           }
         }
+        __threadfence();
+        __syncwarp();
+        if (lane == 0) {
+          cnt_sm[rs] = 0;
+          if (atomicAdd(f.arrive + b, 1) == M - 1) {
+            // this CTA completed bucket b: hand it to the solver warp
+            __threadfence();
+            const int pos = atomicAdd(&q_tail, 1);
+            ((volatile int*)queue_sm)[pos % kFusedQueue] = (int)b;
+            __threadfence_block();
+          }
+        }
+      }
 #pragma unroll
-        for (int i = 0; i < NP; ++i) acc64[i] = 0.0;
-        ++gb;
-        g_open = false;
+      for (int i = 0; i < NP; ++i) acc64[i] = 0.0;
+    } else {
+      // ---- combination of this warp's piece of bucket b, backwards
+      int ok = 0;
+      if (lane == 0) ok = fused_wait(f.ready + b, 1, v.hdr) ? 1 : 0;
+      if (!__shfl_sync(0xffffffffu, ok, 0)) {
+        failed = true;
+        break;
       }
-    }
-
-    // ---- open the combination of bucket cb once its beta is ready
-    if (want) {
-      flag = __shfl_sync(0xffffffffu, flag, 0);
-      bool more = gb < B && gb <= cb + 1;
-      if (more && gb == cb + 1 && g_open) more = g_next < ((g_nv * f.lookahead) >> 10);
-      if (!flag && !more) {   // nothing left to overlap: wait
-        int ok = 0;
-        if (lane == 0) ok = fused_wait(f.ready + cb, 1, v.hdr) ? 1 : 0;
-        if (!__shfl_sync(0xffffffffu, ok, 0)) return;
-        flag = 1;
-      }
-      if (flag) {
-        fence_acquire();
-        float bl = lane < K ? __ldcg(v.beta + cb * K + lane) : 0.0f;
+      fence_acquire();
+      float beta[K];
+      {
+        const float bl = lane < K ? __ldcg(v.beta + b * K + lane) : 0.0f;
 #pragma unroll
         for (int k = 0; k < K; ++k) beta[k] = __shfl_sync(0xffffffffu, bl, k);
-        int64_t lo, hi;
-        warp_piece<EPV>(v, cb, cta, n, wid, &lo, &hi);
-        c_vs = (lo + EPV - 1) / EPV * EPV;
-        if (c_vs > hi) c_vs = hi;
-        int64_t ve = hi / EPV * EPV;
-        if (ve < c_vs) ve = c_vs;
-        c_nv = (ve - c_vs) / EPV;
-        const int nh = (int)(c_vs - lo), nt = (int)(hi - ve);
-        if (lane < nh + nt) {
-          const int64_t idx = lane < nh ? lo + lane : ve + (lane - nh);
-          float t = 0.0f;
-#pragma unroll
-          for (int k = 0; k < K; ++k) t = fmaf(beta[k], load_scalar<DT>(g.p[k], idx), t);
-          store_scalar<DTO>(out, idx, t);
-        }
-        c_next = 0;
-        c_open = true;
-      } else if (*(volatile int32_t*)&v.hdr->status != 0) {
-        return;
       }
-    }
-
-    // ---- one combination step of bucket cb, from the end of the piece back
-    // to its start: the lines the Gram pass read last are read first, so
-    // an LRU L2 still holds them even when the bucket and its output
-    // together slightly exceed the cache
-    if (c_open) {
-      uint4 r[STEP][K];
+      const int nh = q == 0 ? (int)(pc.vs - pc.bo) : 0;
+      const int nt = q == W - 1 ? (int)(pc.be - pc.ve) : 0;
+      if (lane < nh + nt) {
+        const int64_t idx = lane < nh ? pc.bo + lane : pc.ve + (lane - nh);
+        float t = 0.0f;
 #pragma unroll
-      for (int j = 0; j < STEP; ++j) {
-        const int64_t idx = c_nv - 1 - (c_next + lane + 32 * j);
-        if (idx >= 0) {
-#pragma unroll
-          for (int k = 0; k < K; ++k)
-            r[j][k] = ld16_policy(static_cast<const char*>(g.p[k]) + (c_vs + idx * EPV) * IB, last_use);
-        }
+        for (int k = 0; k < K; ++k) t = fmaf(beta[k], load_scalar<DT>(g.p[k], idx), t);
+        store_scalar<DTO>(out, idx, t);
       }
-#pragma unroll
-      for (int j = 0; j < STEP; ++j) {
-        const int64_t idx = c_nv - 1 - (c_next + lane + 32 * j);
-        if (idx >= 0) {
+      for (int64_t i = 0; i < n_items; ++i) {
+        pr.issue(v, g, slot, issued++ % S);
+        cp_async_wait<S - 1>();
+        const int st = consumed++ % S;
+        const int64_t idx = pc.vhi - 1 - (lane + 32 * i);
+        if (idx >= pc.vlo) {
           float y[EPV];
 #pragma unroll
-          for (int q = 0; q < EPV; ++q) {
+          for (int e = 0; e < EPV; ++e) {
             float t = 0.0f;
 #pragma unroll
-            for (int k = 0; k < K; ++k) t = fmaf(beta[k], vec_elem<DT>(r[j][k], q), t);
-            y[q] = t;
+            for (int k = 0; k < K; ++k) t = fmaf(beta[k], vec_elem<DT>(*slot(st, k), e), t);
+            y[e] = t;
           }
-          store_out<DTO>(out, c_vs + idx * EPV, y, EPV);
+          store_out<DTO>(out, pc.vs + idx * EPV, y, EPV);
         }
-      }
-      c_next += 32 * STEP;
-      if (c_next >= c_nv) {
-        c_open = false;
-        ++cb;
       }
     }
   }
+  cp_async_wait<0>();
+  __syncwarp();
+  if (lane == 0) atomicAdd(&done_warps, 1);
 }
 
 #define BKMOO_FUSED_ROW(K, DTI)                                               \

@@ -6,6 +6,7 @@
 // events per call).
 #include <cuda_runtime.h>
 
+#include <cstdlib>
 #include <cstring>
 #include <map>
 #include <mutex>
@@ -80,7 +81,40 @@ const void* fused_fn(int K, int dti, int dto) {
                 : (K <= 6 ? fused_fn_bf16_k5_6(K, dto) : fused_fn_bf16_k7_8(K, dto));
 }
 
-// The fused path: one cooperative (co-resident) launch; the last CTA solves.
+// Fused-path sizing.  The bytes that pass through L2 between a bucket's Gram
+// read and its re-read are about (lookahead + 1) buckets per group, so the
+// group count is the budget over that (at least 1, at most one group per 4
+// CTAs and one per bucket).  The budget is a fraction of L2 (3/4: measured
+// re-reads of more than about 76 MB of 126 MB fall to HBM speed on this
+// part, but a lookahead of one bucket and this budget measured fastest).
+// BKMOO_FUSED_L2_BUDGET (bytes) and BKMOO_FUSED_LOOKAHEAD (buckets) override
+// the defaults.
+struct FusedShape {
+  int n_groups;
+  int lookahead;
+};
+FusedShape fused_shape(int grid, int64_t n_buckets, double bucket_bytes, int l2_bytes) {
+  double budget = 0.75 * (double)l2_bytes;
+  int lookahead = 1;
+  if (const char* e = std::getenv("BKMOO_FUSED_L2_BUDGET")) {
+    const double x = std::atof(e);
+    if (x > 0) budget = x;
+  }
+  if (const char* e = std::getenv("BKMOO_FUSED_LOOKAHEAD")) {
+    const int x = std::atoi(e);
+    if (x >= 0 && x <= kFusedRing - 2) lookahead = x;
+  }
+  double ng = budget / ((lookahead + 1) * (bucket_bytes > 1.0 ? bucket_bytes : 1.0));
+  int64_t n = (int64_t)ng;
+  const int64_t cap = grid / 4 > 0 ? grid / 4 : 1;
+  if (n > cap) n = cap;
+  if (n > n_buckets) n = n_buckets;
+  if (n < 1) n = 1;
+  return FusedShape{(int)n, lookahead};
+}
+
+// The fused path: one cooperative (co-resident) launch of kFusedThreads per
+// CTA, one CTA per SM.
 int launch_fused(const GradPtrs& g, const PlanView& v, const SolveParams& sp, void* ws,
                  float* out_weights, int32_t* out_status, void* out, int dto,
                  double bucket_bytes_max, cudaStream_t s) {
@@ -92,36 +126,31 @@ int launch_fused(const GradPtrs& g, const PlanView& v, const SolveParams& sp, vo
     return BKMOO_ERR_CUDA;
   const void* fn = fused_fn(v.K, v.in_dtype, dto);
   int grid = 0;
-  if (persistent_grid(fn, kThreads, &grid) != cudaSuccess) return BKMOO_ERR_CUDA;
-  if (grid > kFusedMaxCtas + 1) grid = kFusedMaxCtas + 1;
-  if (grid < 2) return BKMOO_ERR_CUDA;
+  if (persistent_grid(fn, kFusedThreads, &grid, fused_smem_bytes(v.K)) != cudaSuccess)
+    return BKMOO_ERR_CUDA;
+  if (grid > kFusedMaxCtas) grid = kFusedMaxCtas;
+  if (grid < 1) return BKMOO_ERR_CUDA;
+  int dev = 0, l2 = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&l2, cudaDevAttrL2CacheSize, dev) != cudaSuccess)
+    return BKMOO_ERR_CUDA;
+  const FusedShape sh = fused_shape(grid, v.n_buckets, bucket_bytes_max, l2);
   FusedView f;
   f.v = v;
-  f.lookahead = 0;
   f.arrive = reinterpret_cast<int32_t*>(base + L.arrive);
   f.ready = reinterpret_cast<int32_t*>(base + L.ready);
   f.ring = reinterpret_cast<double*>(base + L.ring);
   f.out_weights = out_weights;
   f.out_status = out_status;
-  f.n_stream = grid - 1;
-  // Look-ahead that keeps one bucket plus the part of the next one already
-  // read within 90 % of L2 (at least 1/20 of a bucket, at most a whole one).
-  {
-    int dev = 0, l2 = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess ||
-        cudaDeviceGetAttribute(&l2, cudaDevAttrL2CacheSize, dev) != cudaSuccess)
-      return BKMOO_ERR_CUDA;
-    const double wmax = bucket_bytes_max;
-    double la = (0.9 * (double)l2 - wmax) / (wmax > 0 ? wmax : 1.0);
-    if (la < 0.05) la = 0.05;
-    if (la > 1.0) la = 1.0;
-    f.lookahead = (int32_t)(la * 1024.0);
-  }
+  f.n_groups = sh.n_groups;
+  f.group_ctas = (grid + sh.n_groups - 1) / sh.n_groups;
+  f.lookahead = sh.lookahead;
   GradPtrs ga = g;
   SolveParams spa = sp;
   void* outp = out;
   void* args[] = {&ga, &f, &spa, &outp};
-  if (cudaLaunchCooperativeKernel(fn, dim3(grid), dim3(kThreads), args, 0, s) != cudaSuccess)
+  if (cudaLaunchCooperativeKernel(fn, dim3(grid), dim3(kFusedThreads), args,
+                                  fused_smem_bytes(v.K), s) != cudaSuccess)
     return BKMOO_ERR_CUDA;
   return BKMOO_OK;
 }
@@ -188,7 +217,7 @@ int launch_combine(const GradPtrs& g, const PlanView& v, void* out, int32_t out_
                    cudaStream_t s) {
   const int64_t nch = v.c_hi - v.c_lo;
   if (nch <= 0) return BKMOO_OK;
-  const bool pf = BKMOO_COMBINE_PREFETCH && v.K <= 8;
+  const bool pf = BKMOO_COMBINE_PREFETCH != 0;
   const void* fn = pf ? combine_prefetch_fn(v.K, v.in_dtype, out_dtype)
                       : combine_fn(v.K, v.in_dtype, out_dtype);
   const int smem = pf ? combine_prefetch_smem(v.K) : 0;
@@ -405,7 +434,7 @@ int bkmoo_resolve(const void* const* grads, int32_t K, int32_t in_dtype, const i
     for (int64_t b = 0; b < n_buckets; ++b)
       if (offsets[b + 1] - offsets[b] > nmax) nmax = offsets[b + 1] - offsets[b];
     r = launch_fused(g, v, sp, ws, out_weights, out_status, out_dir, out_dtype,
-                     (double)nmax * K * elem_bytes(in_dtype), s);
+                     (double)nmax * (K * elem_bytes(in_dtype) + elem_bytes(out_dtype)), s);
     if (r != BKMOO_OK) return r;
     for (int i = 1; i < 4; ++i)
       if (ev && cudaEventRecord(ev[i], s) != cudaSuccess) return BKMOO_ERR_CUDA;
