@@ -54,7 +54,7 @@ def _args():
                          "against plain gradient accumulation")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--e2e-steps", type=int, default=3)
+    ap.add_argument("--e2e-steps", type=int, default=6)
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     return ap.parse_args()
 
@@ -618,13 +618,79 @@ def e2e_measure(a, w, off, grads, res, params, dev, tdt):
         one()
     dt = (time.perf_counter() - t0) / a.e2e_steps
     gb = w.K * N * w.elem_bytes
+    gbo = N * host_out.element_size()
     r = {"value": gb / dt / GB, "unit": "GB/s", "ms_per_step": dt * 1e3,
-         "h2d_bytes_per_step": gb, "d2h_bytes_per_step": N * host_out.element_size(),
+         "h2d_bytes_per_step": gb, "d2h_bytes_per_step": gbo,
          "steps": a.e2e_steps, "api": "bkmoo_resolve_host",
          "window_elems": window, "staging_bytes": staging.numel(),
-         "link_GBps": (gb + N * host_out.element_size()) / dt / GB}
+         "link_GBps": (gb + gbo) / dt / GB}
+    del staging
+    link = link_bound(host, host_out, window, dev, reps=max(2, a.e2e_steps // 2))
+    r["link_bound"] = link
+    r["ms_over_link_bound"] = dt * 1e3 / link["both_ms"]
+    r["ms_over_one_way_h2d"] = dt * 1e3 / link["h2d_only_ms"]
     if sample:
         r["sample"] = sample
+    return r
+
+
+def link_bound(host, host_out, window, dev, reps=2):
+    """What the host link itself allows for the end-to-end step, measured on
+    the same page-locked buffers with the same window length: every input
+    window copied host -> device into one of two device slots (one stream),
+    every output window copied device -> host (another stream), each alone
+    and both at once (window w's input beside window w-1's output).  No
+    kernel runs; the slots' contents are discarded."""
+    import torch
+
+    K, N = len(host), host[0].numel()
+    slots = [[torch.empty(window, dtype=host[0].dtype, device=dev) for _ in range(K)]
+             for _ in range(2)]
+    outs = [torch.empty(window, dtype=host_out.dtype, device=dev) for _ in range(2)]
+    s_in, s_out = torch.cuda.Stream(dev), torch.cuda.Stream(dev)
+    wins = [(lo, min(lo + window, N)) for lo in range(0, N, window)]
+
+    def h2d(i, lo, hi):
+        with torch.cuda.stream(s_in):
+            for k in range(K):
+                slots[i % 2][k][:hi - lo].copy_(host[k][lo:hi], non_blocking=True)
+
+    def d2h(i, lo, hi):
+        with torch.cuda.stream(s_out):
+            host_out[lo:hi].copy_(outs[i % 2][:hi - lo], non_blocking=True)
+
+    def timed(fn):
+        best = None
+        for _ in range(reps):
+            torch.cuda.synchronize(dev)
+            t0 = time.perf_counter()
+            fn()
+            torch.cuda.synchronize(dev)
+            t = time.perf_counter() - t0
+            best = t if best is None else min(best, t)
+        return best * 1e3
+
+    def only_in():
+        for i, (lo, hi) in enumerate(wins):
+            h2d(i, lo, hi)
+
+    def only_out():
+        for i, (lo, hi) in enumerate(wins):
+            d2h(i, lo, hi)
+
+    def both():
+        for i, (lo, hi) in enumerate(wins):
+            h2d(i, lo, hi)
+            if i:
+                d2h(i - 1, *wins[i - 1])
+        d2h(len(wins) - 1, *wins[-1])
+
+    r = {"h2d_only_ms": timed(only_in), "d2h_only_ms": timed(only_out), "both_ms": timed(both)}
+    gb_in = sum(t.numel() * t.element_size() for t in host)
+    r["h2d_GBps"] = gb_in / r["h2d_only_ms"] * 1e3 / GB
+    r["d2h_GBps"] = host_out.numel() * host_out.element_size() / r["d2h_only_ms"] * 1e3 / GB
+    r["reps"] = reps
+    del slots, outs
     return r
 
 
