@@ -95,14 +95,46 @@ struct BucketTracker {
 
 // This thread's sequence of 16-byte positions: chunk w = c_lo + blockIdx.x,
 // + gridDim.x, ...; within a chunk the vectors i = t, t + 256, ... < nv.
+// On entering a chunk the cursor also issues the loads of the bounds of the
+// bucket its next chunk is guessed to fall in (from the current bucket's
+// chunk count), so that the next move finds them in registers instead of
+// waiting a round trip on the path of the copies; a wrong guess falls back
+// to BucketTracker::seek.
 template <int EPV>
 struct VecCursor {
   BucketTracker bt;
   int64_t w, vs;
   int nv, i;
+  int64_t nb, n0, n1, p0, p1;   // preloaded guess for the next chunk (nb < 0: none)
+  __device__ void preload(const PlanView& v) {
+    nb = -1;
+    const int64_t wn = w + gridDim.x;
+    if (wn < bt.c1 || wn >= v.c_hi) return;
+    const int64_t g = bt.b + (wn - bt.c0) / (bt.c1 - bt.c0);
+    if (g >= v.n_buckets) return;
+    nb = g;
+    n0 = v.chunk_prefix[g];
+    n1 = v.chunk_prefix[g + 1];
+    p0 = v.offsets[g];
+    p1 = v.offsets[g + 1];
+  }
+  __device__ void move(const PlanView& v) {
+    if (!(bt.c0 <= w && w < bt.c1)) {
+      if (nb >= 0 && n0 <= w && w < n1) {
+        bt.b = nb;
+        bt.c0 = n0;
+        bt.c1 = n1;
+        bt.o0 = p0;
+        bt.o1 = p1;
+      } else {
+        bt.seek(v, w);
+      }
+    }
+    preload(v);
+  }
   __device__ void settle(const PlanView& v) {
     while (w < v.c_hi) {
-      bt.seek(v, w);
+      move(v);
       int64_t s, e;
       bt.range<EPV>(v, w, &s, &e, &vs, &nv);
       if (i < nv) return;
@@ -113,13 +145,18 @@ struct VecCursor {
   __device__ void begin(const PlanView& v) {
     w = v.c_lo + blockIdx.x;
     bt.init(v);
+    nb = -1;
     i = threadIdx.x;
     settle(v);
   }
   __device__ bool more(const PlanView& v) const { return w < v.c_hi; }
   __device__ void next(const PlanView& v) {
     i += kThreads;
-    if (i >= nv) settle(v);
+    if (i >= nv) {
+      w += gridDim.x;
+      i = threadIdx.x;
+      settle(v);
+    }
   }
 };
 
@@ -162,7 +199,9 @@ __global__ void __launch_bounds__(kThreads) gram_prefetch_kernel(const GradPtrs 
   BucketTracker ct;
   ct.init(v);
   for (int64_t w = v.c_lo + blockIdx.x; w < v.c_hi; w += gridDim.x) {
-    ct.seek(v, w);
+    // the producer is usually still on this chunk: take its bucket bounds
+    if (pc.w == w) ct = pc.bt;
+    else ct.seek(v, w);
     int64_t s0, e, vs;
     int nv;
     ct.range<EPV>(v, w, &s0, &e, &vs, &nv);
