@@ -17,10 +17,12 @@ namespace bkmoo {
 #endif
 constexpr int kCombinePrefetchStages = BKMOO_COMBINE_PREFETCH_STAGES;
 
-// Stages per thread: 4 for K <= 8; 3 above (K = 16: 192 KB of slots, one
-// CTA per SM with 128 KB of copies in flight).
+// Stages per thread (measured on GB300): 2 for K <= 4 (Qwen3-8B K=4 bf16
+// combination 11.96 -> 11.83 ms against 4 stages; sweep K=2 1.80 -> 1.77 ms),
+// 4 for K = 5..8 (Llama-3.2-1B K=8: 3.11 ms, 3.20 with 2 stages), 3 above
+// (K = 16: 192 KB of slots, one CTA per SM with 128 KB of copies in flight).
 __host__ __device__ constexpr int combine_prefetch_stages(int K) {
-  return K <= 8 ? kCombinePrefetchStages : 3;
+  return K <= 4 ? 2 : K <= 8 ? kCombinePrefetchStages : 3;
 }
 __host__ __device__ constexpr int combine_prefetch_smem_bytes(int K) {
   return combine_prefetch_stages(K) * K * kThreads * 16;
