@@ -67,7 +67,7 @@ namespace bkmoo {
 constexpr uint64_t kFusedWaitNs = 1000000000ull;  // a wait gives up after 1 s
 constexpr int kFusedQueue = 16;                    // solver queue entries per CTA
 
-// L2 eviction-priority policies (createpolicy) and 16-byte loads carrying them.
+// L2 eviction-priority policies (createpolicy).
 __device__ __forceinline__ uint64_t policy_evict_last() {
   uint64_t pol;
   asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(pol));
@@ -78,19 +78,12 @@ __device__ __forceinline__ uint64_t policy_evict_first() {
   asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(pol));
   return pol;
 }
-__device__ __forceinline__ uint4 ld16_policy_nc(const void* p, uint64_t pol) {
-  uint4 r;
-  asm volatile("ld.global.nc.L1::no_allocate.L2::cache_hint.v4.u32 {%0,%1,%2,%3}, [%4], %5;"
-               : "=r"(r.x), "=r"(r.y), "=r"(r.z), "=r"(r.w)
-               : "l"(p), "l"(pol));
-  return r;
-}
-__device__ __forceinline__ uint4 ld16_policy(const void* p, uint64_t pol) {
-  uint4 r;
-  asm volatile("ld.global.L1::no_allocate.L2::cache_hint.v4.u32 {%0,%1,%2,%3}, [%4], %5;"
-               : "=r"(r.x), "=r"(r.y), "=r"(r.z), "=r"(r.w)
-               : "l"(p), "l"(pol));
-  return r;
+// cp.async of 16 bytes carrying an L2 eviction policy.
+__device__ __forceinline__ void cp_async16_policy(void* smem_dst, const void* src, uint64_t pol) {
+  asm volatile("cp.async.cg.shared.global.L2::cache_hint [%0], [%1], 16, %2;" ::"r"(
+                   (uint32_t)__cvta_generic_to_shared(smem_dst)),
+               "l"(src), "l"(pol)
+               : "memory");
 }
 
 __device__ __forceinline__ int ld_acquire(const int32_t* p) {
@@ -329,9 +322,13 @@ struct FusedProducer {
     if (seg < sch.total()) {
       const int64_t idx = comb ? hi - 1 - (lane + 32 * item) : lo + lane + 32 * item;
       if (idx >= lo && idx < hi) {
+        // Gram reads stay in L2 for the re-read (evict_last); the re-read
+        // is the last use (evict_first)
+        const uint64_t pol = comb ? policy_evict_first() : policy_evict_last();
         const int64_t off = (vs + idx * EPV) * IB;
 #pragma unroll
-        for (int k = 0; k < K; ++k) cp_async16(slot(stage, k), static_cast<const char*>(g.p[k]) + off);
+        for (int k = 0; k < K; ++k)
+          cp_async16_policy(slot(stage, k), static_cast<const char*>(g.p[k]) + off, pol);
       }
       if (++item == n_items) {
         ++seg;
