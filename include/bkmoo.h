@@ -303,12 +303,12 @@ int bkmoo_host_staging_size(int32_t K, int32_t in_dtype, int32_t out_dtype,
  * send its direction on and free the bucket's device copy -- so that device
  * memory holds only a bounded window of buckets, not the K full gradients.
  *
- * Buckets go through two device staging slots in windows of whole buckets:
+ * Buckets go through three device staging slots in windows of whole buckets:
  * while window w is resolved (Gram -> rule -> combination on `stream`, the
  * same kernels and the same per-chunk arithmetic as bkmoo_resolve, so beta
- * and the direction are bit-identical to it), window w+1 is copied in and
- * window w-1's direction copied out on two internal copy streams, created
- * and destroyed by the call.  Work already queued on `stream` comes first;
+ * and the direction are bit-identical to it), the next windows are copied
+ * in and earlier windows' directions copied out on two internal copy
+ * streams, created and destroyed by the call.  Work already queued on `stream` comes first;
  * `stream` completes only after the last byte reaches host_out.
  *
  * host_grads: host array of K host pointers (16-byte aligned), N elements
@@ -319,7 +319,7 @@ int bkmoo_host_staging_size(int32_t K, int32_t in_dtype, int32_t out_dtype,
  * out_weights, out_status, ws, ws_bytes, rule, p: as in bkmoo_resolve (device
  *   buffers; ws initialised for this plan).  p->events and
  *   BKMOO_FLAG_FUSED are ignored.
- * staging: device, 256-byte aligned, staging_bytes long.  It holds two
+ * staging: device, 256-byte aligned, staging_bytes long.  It holds three
  *   slots of K input regions and one output region of
  *   round_up(cap e + 16, 256) bytes each (e the region's element size); cap,
  *   the window length in elements per language, is the largest that fits.

@@ -157,13 +157,13 @@ def test_resolve_rejects_bad_arguments_without_launch():
 
 
 def test_host_staging_size():
-    """Two slots, each K input regions and one output region of the largest
+    """Three slots, each K input regions and one output region of the largest
     of (window, longest bucket) elements plus 16 bytes, 256-byte aligned."""
     off = np.array([0, 1000, 2500, 2600], dtype=np.int64)
 
     def expect(K, ei, eo, n):
         r = lambda e: (n * e + 16 + 255) // 256 * 256
-        return 2 * (K * r(ei) + r(eo))
+        return 3 * (K * r(ei) + r(eo))
 
     assert bk.bkmoo_host_staging_size(4, bk.BKMOO_BF16, bk.BKMOO_BF16, off) == expect(4, 2, 2, 1500)
     assert bk.bkmoo_host_staging_size(3, bk.BKMOO_F32, bk.BKMOO_BF16, off, 10**6) == \

@@ -1,5 +1,5 @@
 """GPU: bkmoo_resolve_host (gradients and direction in host memory, buckets
-streamed through two device staging slots) against the device-resident
+streamed through three device staging slots) against the device-resident
 bkmoo_resolve -- bit-identical beta, status and direction -- and against the
 fp64 oracle, with windows of one and of several buckets, ragged and unaligned
 bucket starts, in-place use and page-locked and pageable host buffers."""
