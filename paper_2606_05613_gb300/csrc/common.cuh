@@ -305,6 +305,17 @@ const void* fused_fn_bf16_k1_4(int K, int dtype_out);
 const void* fused_fn_bf16_k5_6(int K, int dtype_out);
 const void* fused_fn_bf16_k7_8(int K, int dtype_out);
 
+// Cluster-per-bucket fused kernels (fused_cluster.cu), K <= kClusterMaxK,
+// signature (GradPtrs, PlanView, SolveParams, float* out_weights,
+// int32_t* out_status, void* out), clusters of 8 CTAs of 256 threads with
+// fused_cluster_smem(K) bytes of dynamic shared memory.
+constexpr int kClusterMaxK = 4;
+constexpr int kClusterCtas = 8;
+constexpr int kClusterWarps = 16;
+constexpr int kClusterThreads = 32 * kClusterWarps;
+const void* fused_cluster_fn(int K, int dti, int dto);
+int fused_cluster_smem(int K);
+
 // solve.cu
 cudaError_t launch_solve(const PlanView& v, const SolveParams& p, float* out_weights,
                          int32_t* out_status, cudaStream_t s);

@@ -289,50 +289,67 @@ struct FusedSched {
   }
 };
 
-// Per-lane producer: walks the same segments as the consumer and copies
+// Per-thread producer: walks the same segments as the consumer and copies
 // the K vectors of its next item into stage (issued % S) with cp.async;
-// every call commits one group (empty once the schedule is exhausted).
-// Items of a segment: n = ceil(piece vectors / 32) per lane (warp-uniform);
-// item i is vector lo + lane + 32 i of a Gram piece, hi - 1 - (lane + 32 i)
-// of a combination piece (read backwards), valid when inside [lo, hi).
-template <int K, int DT>
+// every call commits one group (empty once the schedule is exhausted).  A
+// piece is shared by STRIDE threads (a warp here; a whole CTA in the
+// cluster kernel).  Items of a segment: n = ceil(piece vectors / STRIDE) per
+// thread (uniform over the STRIDE threads); item i is vector
+// lo + lane + STRIDE i of a Gram piece, hi - 1 - (lane + STRIDE i) of a
+// combination piece (read backwards), valid when inside [lo, hi).
+template <int K, int DT, int STRIDE = 32>
 struct FusedProducer {
   FusedSched sch;
-  int64_t seg, vs, lo, hi, item, n_items;
-  bool comb;
-  int grp, ng, q, W, lane;
-  __device__ void open(const PlanView& v) {
-    while (seg < sch.total()) {
+  int64_t seg, total;
+  int grp, ng, q, W, lane;   // lane: this thread's index among the STRIDE that share a piece
+  const char* src[K];        // this thread's next item in each gradient
+  int64_t step;              // bytes to its following item (negative: backwards)
+  int left, valid;           // items left in the segment, and how many of them are valid
+  uint64_t pol;
+  __device__ void begin(const PlanView& v, const GradPtrs& g) {
+    total = sch.total();
+    seg = 0;
+    open(v, g);
+  }
+  __device__ void open(const PlanView& v, const GradPtrs& g) {
+    constexpr int EPV = elems_per_vec(DT);
+    constexpr int IB = 16 / EPV;
+    while (seg < total) {
+      bool comb;
       int64_t j;
       sch.seg_at(seg, &comb, &j);
-      const Piece pc = fused_piece<elems_per_vec(DT)>(v, grp + j * ng, q, W);
-      vs = pc.vs;
-      lo = pc.vlo;
-      hi = pc.vhi;
-      n_items = (hi - lo + 31) / 32;
-      item = 0;
-      if (n_items > 0) return;
+      const Piece pc = fused_piece<EPV>(v, grp + j * ng, q, W);
+      const int64_t n = pc.vhi - pc.vlo;
+      left = (int)((n + STRIDE - 1) / STRIDE);
+      valid = n > lane ? (int)((n - lane + STRIDE - 1) / STRIDE) : 0;
+      // pointers are only dereferenced for the `valid` first items
+      const int64_t first = comb ? pc.vhi - 1 - lane : pc.vlo + lane;
+      step = (comb ? -(int64_t)STRIDE : (int64_t)STRIDE) * 16;
+#pragma unroll
+      for (int k = 0; k < K; ++k)
+        src[k] = static_cast<const char*>(g.p[k]) + (pc.vs + first * EPV) * IB;
+      // Gram reads stay in L2 for the re-read (evict_last); the re-read is
+      // the last use (evict_first)
+      pol = comb ? policy_evict_first() : policy_evict_last();
+      if (left > 0) return;
       ++seg;
     }
   }
   template <typename Slot>
-  __device__ void issue(const PlanView& v, const GradPtrs& g, Slot slot, int stage) {
-    constexpr int EPV = elems_per_vec(DT);
-    constexpr int IB = 16 / EPV;
-    if (seg < sch.total()) {
-      const int64_t idx = comb ? hi - 1 - (lane + 32 * item) : lo + lane + 32 * item;
-      if (idx >= lo && idx < hi) {
-        // Gram reads stay in L2 for the re-read (evict_last); the re-read
-        // is the last use (evict_first)
-        const uint64_t pol = comb ? policy_evict_first() : policy_evict_last();
-        const int64_t off = (vs + idx * EPV) * IB;
+  __device__ __forceinline__ void issue(const PlanView& v, const GradPtrs& g, Slot slot,
+                                        int stage) {
+    if (seg < total) {
+      if (valid > 0) {
 #pragma unroll
-        for (int k = 0; k < K; ++k)
-          cp_async16_policy(slot(stage, k), static_cast<const char*>(g.p[k]) + off, pol);
+        for (int k = 0; k < K; ++k) {
+          cp_async16_policy(slot(stage, k), src[k], pol);
+          src[k] += step;
+        }
+        --valid;
       }
-      if (++item == n_items) {
+      if (--left == 0) {
         ++seg;
-        open(v);
+        open(v, g);
       }
     }
     cp_async_commit();
@@ -375,9 +392,11 @@ __global__ void __launch_bounds__(kFusedThreads, 1)
     return;
   }
 
-  // this lane's stage slots: [S][K] 16-byte vectors
-  uint4* my_slots = reinterpret_cast<uint4*>(fused_smem) + (size_t)threadIdx.x * S * K;
-  auto slot = [&](int st, int k) -> uint4* { return my_slots + st * K + k; };
+  // stage slots [S][K][streaming threads] of 16-byte vectors: neighbouring
+  // lanes use neighbouring 16-byte words (no shared-memory bank conflicts)
+  uint4* slots = reinterpret_cast<uint4*>(fused_smem);
+  constexpr int NT = 32 * kFusedStreamWarps;
+  auto slot = [&](int st, int k) -> uint4* { return slots + (st * K + k) * NT + threadIdx.x; };
 
   const int ng = f.n_groups;
   const int cta = blockIdx.x, grp = cta % ng, c_loc = cta / ng;
@@ -388,13 +407,12 @@ __global__ void __launch_bounds__(kFusedThreads, 1)
 
   FusedProducer<K, DT> pr;
   pr.sch = sch;
-  pr.seg = 0;
   pr.grp = grp;
   pr.ng = ng;
   pr.q = q;
   pr.W = W;
   pr.lane = lane;
-  pr.open(v);
+  pr.begin(v, g);
   int issued = 0;
 #pragma unroll 1
   for (int j = 0; j < S - 1; ++j) pr.issue(v, g, slot, issued++ % S);

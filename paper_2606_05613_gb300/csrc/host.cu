@@ -155,6 +155,61 @@ int launch_fused(const GradPtrs& g, const PlanView& v, const SolveParams& sp, vo
   return BKMOO_OK;
 }
 
+// The cluster-per-bucket fused path: as many clusters of kClusterCtas CTAs
+// as can be resident at once (clusters never wait for one another).
+int launch_fused_cluster(const GradPtrs& g, const PlanView& v, const SolveParams& sp,
+                         float* out_weights, int32_t* out_status, void* out, int dto,
+                         cudaStream_t s) {
+  if (cudaMemsetAsync(&v.hdr->status, 0, sizeof(int32_t), s) != cudaSuccess) return BKMOO_ERR_CUDA;
+  if (v.n_buckets == 0) return BKMOO_OK;
+  const void* fn = fused_cluster_fn(v.K, v.in_dtype, dto);
+  if (!fn) return BKMOO_ERR_INVALID;
+  const int smem = fused_cluster_smem(v.K);
+  static std::mutex mu;
+  static std::map<std::pair<int, const void*>, int> clusters;
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return BKMOO_ERR_CUDA;
+  int ncl = 0;
+  {
+    std::lock_guard<std::mutex> lk(mu);
+    auto key = std::make_pair(dev, fn);
+    auto it = clusters.find(key);
+    if (it == clusters.end()) {
+      if (cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) !=
+          cudaSuccess)
+        return BKMOO_ERR_CUDA;
+      cudaLaunchConfig_t cfg = {};
+      cudaLaunchAttribute attr[1];
+      attr[0].id = cudaLaunchAttributeClusterDimension;
+      attr[0].val.clusterDim.x = kClusterCtas;
+      attr[0].val.clusterDim.y = 1;
+      attr[0].val.clusterDim.z = 1;
+      cfg.gridDim = dim3(kClusterCtas);
+      cfg.blockDim = dim3(kClusterThreads);
+      cfg.dynamicSmemBytes = (size_t)smem;
+      cfg.attrs = attr;
+      cfg.numAttrs = 1;
+      int n = 0;
+      if (cudaOccupancyMaxActiveClusters(&n, fn, &cfg) != cudaSuccess) return BKMOO_ERR_CUDA;
+      it = clusters.emplace(key, n).first;
+    }
+    ncl = it->second;
+  }
+  if (ncl < 1) return BKMOO_ERR_CUDA;
+  if ((int64_t)ncl > v.n_buckets) ncl = (int)v.n_buckets;
+  GradPtrs ga = g;
+  PlanView va = v;
+  SolveParams spa = sp;
+  float* ow = out_weights;
+  int32_t* os = out_status;
+  void* outp = out;
+  void* args[] = {&ga, &va, &spa, &ow, &os, &outp};
+  if (cudaLaunchKernel(fn, dim3(ncl * kClusterCtas), dim3(kClusterThreads), args, (size_t)smem,
+                       s) != cudaSuccess)
+    return BKMOO_ERR_CUDA;
+  return BKMOO_OK;
+}
+
 // Common checks of bkmoo_gram / bkmoo_resolve; fills the plan view.
 int prepare(const void* const* grads, int32_t K, int32_t dt, const int64_t* offsets,
             int64_t B, void* ws, size_t ws_bytes, PlanView* v, GradPtrs* g) {
@@ -430,6 +485,16 @@ int bkmoo_resolve(const void* const* grads, int32_t K, int32_t in_dtype, const i
   cudaEvent_t* ev = static_cast<cudaEvent_t*>(prm.events);
   const SolveParams sp = solve_params(rule, prm);
   if (ev && cudaEventRecord(ev[0], s) != cudaSuccess) return BKMOO_ERR_CUDA;
+  const char* fk = std::getenv("BKMOO_FUSED_KERNEL");
+  const bool groups_only = fk && std::strcmp(fk, "groups") == 0;
+  if ((prm.flags & BKMOO_FLAG_FUSED) && K <= kClusterMaxK && !groups_only &&
+      !(prm.flags & BKMOO_FLAG_TEST_WITHHOLD)) {
+    r = launch_fused_cluster(g, v, sp, out_weights, out_status, out_dir, out_dtype, s);
+    if (r != BKMOO_OK) return r;
+    for (int i = 1; i < 4; ++i)
+      if (ev && cudaEventRecord(ev[i], s) != cudaSuccess) return BKMOO_ERR_CUDA;
+    return BKMOO_OK;
+  }
   if ((prm.flags & BKMOO_FLAG_FUSED) && K <= kFusedMaxK) {
     int64_t nmax = 0;
     for (int64_t b = 0; b < n_buckets; ++b)
