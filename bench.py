@@ -45,9 +45,9 @@ def _args():
                     help="qwen3-8b | llama3.2-1b | gpt2-small | tiny | sweep-K-MiB[-<n>M]; "
                          "append -global for one bucket over every parameter")
     ap.add_argument("--rule", default="mgda", choices=["mgda", "pcgrad", "cagrad", "mean"])
-    ap.add_argument("--path", default="3pass", choices=["fused", "3pass"],
-                    help="fused: one persistent launch per step (re-read from L2); "
-                         "3pass: Gram, solve and combination launches")
+    ap.add_argument("--path", default="auto", choices=["auto", "fused", "3pass"],
+                    help="auto: the library's per-plan choice; fused: one launch per step "
+                         "(re-read from L2); 3pass: Gram, solve and combination launches")
     ap.add_argument("--hook", action="store_true",
                     help="time a synthetic training step of a GPT-2-small-shaped transformer "
                          "with the per-bucket resolve inside the backward pass (BucketMOO) "
@@ -454,9 +454,13 @@ def main():
     params = bk.bkmoo_default_params()
     if w.max_iter != 256:
         params.max_iter = w.max_iter
-    fused = a.path == "fused"
-    if fused:
+    if a.path == "fused":
         params.flags |= bk.BKMOO_FLAG_FUSED
+    elif a.path == "3pass":
+        params.flags |= bk.BKMOO_FLAG_THREE_PASS
+    path_id = bk.bkmoo_resolve_path(w.K, bk.BKMOO_F32 if tdt == torch.float32 else bk.BKMOO_BF16,
+                                    a.rule, off, params.flags)
+    fused = path_id != 0
 
     def step(evs=None):
         if evs is not None:
@@ -532,9 +536,12 @@ def main():
         "config": dict(base_config(w, off, a.rule),
                        l2="inputs (%.1f GB) >> L2, no flush" % (grad_bytes / GB),
                        parallelism="replicas" if world > 1 else "1 GPU",
-                       path=("fused: one persistent launch per step, combination re-reads "
-                             "each bucket from L2" if fused else
-                             "gram -> solve -> combine (3 launches)")),
+                       path=({1: "fused: one launch, a thread-block cluster per bucket, "
+                                    "combination re-reads each bucket from L2",
+                              2: "fused: one persistent launch, groups of CTAs per bucket, "
+                                 "combination re-reads each bucket from L2"}.get(
+                                  path_id, "gram -> solve -> combine (3 launches)")
+                             + (" (chosen per plan)" if a.path == "auto" else ""))),
         "roofline": roofline,
         "step_roofline": {"bytes_2k1": step_bytes_2k1, "bytes_k1": step_bytes_k1,
                           "frac_2k1_of_measured": step_bytes_2k1 / (ms_step * 1e-3) / GB / peak,

@@ -73,21 +73,30 @@ typedef enum { BKMOO_F32 = 0, BKMOO_BF16 = 1 } bkmoo_dtype;
 #define BKMOO_FLAG_POLISH 0x2u         /* exact active-set completion after
                                           the Frank-Wolfe phase (MGDA and
                                           CAGrad)                            */
-#define BKMOO_FLAG_FUSED 0x4u          /* one persistent launch that resolves
-                                          bucket after bucket while the
-                                          bucket is still in L2 (K <= 8; for
-                                          larger K the flag is ignored and
-                                          the three-pass path runs).  On a
-                                          GB300 it measured slower than the
-                                          three-pass default everywhere: the
-                                          per-bucket solve and hand-offs
-                                          take longer than L2 can hold the
-                                          data streamed meanwhile.  Results
-                                          agree with the three-pass path to
+#define BKMOO_FLAG_FUSED 0x4u          /* one launch that resolves bucket
+                                          after bucket while the bucket is
+                                          still in L2: a thread-block cluster
+                                          per bucket for K <= 4, groups of
+                                          CTAs for K = 5..8; above, ignored
+                                          (three passes).  On a GB300 the
+                                          cluster kernel is faster than three
+                                          passes for K = 4 with 2-8 MiB
+                                          buckets (the per-plan choice takes
+                                          it there, see bkmoo_resolve_path),
+                                          slower for small buckets, large
+                                          buckets and K = 8.  Results agree
+                                          with the three-pass path to
                                           rounding, not bit for bit.         */
+#define BKMOO_FLAG_THREE_PASS 0x8u     /* always the three-launch path (Gram,
+                                          solve, combination); without it and
+                                          without BKMOO_FLAG_FUSED the path is
+                                          chosen per plan, see
+                                          bkmoo_resolve_path                 */
 #define BKMOO_FLAG_TEST_WITHHOLD 0x100u /* testing failure detection, with
-                                          BKMOO_FLAG_FUSED only: the fused
-                                          kernel never publishes bucket 0's
+                                          BKMOO_FLAG_FUSED only (it selects
+                                          the grid-synchronised fused
+                                          kernel): that kernel never
+                                          publishes bucket 0's
                                           coefficients, so its bounded waits
                                           (about 1 s) run out and the call
                                           ends with BKMOO_ERR_TIMEOUT in the
@@ -256,6 +265,9 @@ int bkmoo_gram_noalloc(const void* const* grads, int32_t K, int32_t in_dtype,
  *   BKMOO_ERR_WORKSPACE; or NULL.
  * ws / ws_bytes: the workspace after bkmoo_workspace_init with the same
  *   K, in_dtype and offsets.
+ * Path: three launches (Gram, solve, combination) or one fused launch, as
+ *   bkmoo_resolve_path gives for the plan, rule and p->flags.  Each path is
+ *   deterministic; the two agree to rounding.
  * Returns BKMOO_OK once the work is queued on `stream`.
  */
 int bkmoo_resolve(const void* const* grads, int32_t K, int32_t in_dtype,
@@ -277,7 +289,8 @@ int bkmoo_resolve(const void* const* grads, int32_t K, int32_t in_dtype,
  * elements of out_dir, the rows of out_weights / out_status and the
  * workspace partials of other buckets are not touched, so calls for disjoint
  * bucket ranges may run concurrently on different streams.  Results are
- * bit-identical to bkmoo_resolve's for the same buckets.  The workspace
+ * bit-identical to those of bkmoo_resolve's three-launch path for the same
+ * buckets.  The workspace
  * status word is not cleared (other calls may be in flight); device-side
  * errors are recorded into it.  BKMOO_FLAG_FUSED and p->events are ignored.
  */
@@ -305,8 +318,9 @@ int bkmoo_host_staging_size(int32_t K, int32_t in_dtype, int32_t out_dtype,
  *
  * Buckets go through three device staging slots in windows of whole buckets:
  * while window w is resolved (Gram -> rule -> combination on `stream`, the
- * same kernels and the same per-chunk arithmetic as bkmoo_resolve, so beta
- * and the direction are bit-identical to it), the next windows are copied
+ * same kernels and the same per-chunk arithmetic as bkmoo_resolve's
+ * three-launch path, so beta and the direction are bit-identical to it),
+ * the next windows are copied
  * in and earlier windows' directions copied out on two internal copy
  * streams, created and destroyed by the call.  Work already queued on `stream` comes first;
  * `stream` completes only after the last byte reaches host_out.
@@ -342,6 +356,24 @@ int bkmoo_resolve_host(const void* const* host_grads, int32_t K, int32_t in_dtyp
  * BKMOO_ERR_TIMEOUT).  Writes *status.
  */
 int bkmoo_workspace_status(const void* ws, void* stream, int32_t* status);
+
+/*
+ * bkmoo_resolve_path -- which path bkmoo_resolve takes for this plan, rule
+ * and flags: *path = 0 for the three launches (Gram, solve, combination), 1
+ * for the cluster-per-bucket fused kernel (one bucket per thread-block
+ * cluster, its re-read served from L2), 2 for the grid-synchronised fused
+ * kernel.  BKMOO_FLAG_THREE_PASS gives 0; BKMOO_FLAG_FUSED gives 1 for
+ * K <= 4 (2 with BKMOO_FLAG_TEST_WITHHOLD), 2 for K = 5..8, 0 above.
+ * Without either flag the choice follows measurements on GB300 (sweeps of
+ * 1e9 fp32 and 2e9 bf16 elements per language): 1 when K = 4, the rule is
+ * not CAGrad (whose per-bucket solve is too long to hide), the largest
+ * bucket holds 2-8 MiB per language for fp32 gradients or 4-8 MiB for bf16,
+ * and at least 90 % of the elements lie in buckets of at least half that
+ * size; 0 otherwise.  Host only; BKMOO_ERR_INVALID on bad arguments.
+ * bkmoo_resolve_buckets and bkmoo_resolve_host always take path 0.
+ */
+int bkmoo_resolve_path(int32_t K, int32_t in_dtype, int32_t rule, const int64_t* offsets,
+                       int64_t n_buckets, uint32_t flags, int32_t* path);
 
 /* Static English text for a bkmoo_status value. */
 const char* bkmoo_status_string(int32_t status);

@@ -210,6 +210,34 @@ int launch_fused_cluster(const GradPtrs& g, const PlanView& v, const SolveParams
   return BKMOO_OK;
 }
 
+// Path of bkmoo_resolve (see bkmoo_resolve_path in bkmoo.h): 0 three
+// launches, 1 cluster-per-bucket fused kernel, 2 grid-synchronised fused
+// kernel.
+int choose_path(int32_t K, int32_t dt, int32_t rule, const int64_t* off, int64_t B,
+                uint32_t flags) {
+  if (flags & BKMOO_FLAG_THREE_PASS) return 0;
+  if (flags & BKMOO_FLAG_FUSED) {
+    if (K <= kClusterMaxK && !(flags & BKMOO_FLAG_TEST_WITHHOLD)) {
+      const char* fk = std::getenv("BKMOO_FUSED_KERNEL");
+      if (!(fk && std::strcmp(fk, "groups") == 0)) return 1;
+    }
+    return K <= kFusedMaxK ? 2 : 0;
+  }
+  // measured on GB300: the cluster kernel is faster only for K = 4 with
+  // mid-sized buckets (MGDA 4.69 vs 5.07 ms at 2 MiB fp32, 4.83 vs 5.01 ms at
+  // 4 MiB bf16; MEAN and PCGrad more, CAGrad slower)
+  if (K != 4 || rule == BKMOO_CAGRAD || B < 1) return 0;
+  int64_t smax = 0;
+  for (int64_t b = 0; b < B; ++b) smax = off[b + 1] - off[b] > smax ? off[b + 1] - off[b] : smax;
+  const double bytes = (double)smax * elem_bytes(dt), mib = 1024.0 * 1024.0;
+  const double lo = (dt == BKMOO_F32 ? 2.0 : 4.0) * mib, hi = 8.0 * mib;
+  if (bytes < lo || bytes > hi) return 0;
+  int64_t big = 0;
+  for (int64_t b = 0; b < B; ++b)
+    if (2 * (off[b + 1] - off[b]) >= smax) big += off[b + 1] - off[b];
+  return big * 10 >= off[B] * 9 ? 1 : 0;
+}
+
 // Common checks of bkmoo_gram / bkmoo_resolve; fills the plan view.
 int prepare(const void* const* grads, int32_t K, int32_t dt, const int64_t* offsets,
             int64_t B, void* ws, size_t ws_bytes, PlanView* v, GradPtrs* g) {
@@ -485,17 +513,15 @@ int bkmoo_resolve(const void* const* grads, int32_t K, int32_t in_dtype, const i
   cudaEvent_t* ev = static_cast<cudaEvent_t*>(prm.events);
   const SolveParams sp = solve_params(rule, prm);
   if (ev && cudaEventRecord(ev[0], s) != cudaSuccess) return BKMOO_ERR_CUDA;
-  const char* fk = std::getenv("BKMOO_FUSED_KERNEL");
-  const bool groups_only = fk && std::strcmp(fk, "groups") == 0;
-  if ((prm.flags & BKMOO_FLAG_FUSED) && K <= kClusterMaxK && !groups_only &&
-      !(prm.flags & BKMOO_FLAG_TEST_WITHHOLD)) {
+  const int path = choose_path(K, in_dtype, rule, offsets, n_buckets, prm.flags);
+  if (path == 1) {
     r = launch_fused_cluster(g, v, sp, out_weights, out_status, out_dir, out_dtype, s);
     if (r != BKMOO_OK) return r;
     for (int i = 1; i < 4; ++i)
       if (ev && cudaEventRecord(ev[i], s) != cudaSuccess) return BKMOO_ERR_CUDA;
     return BKMOO_OK;
   }
-  if ((prm.flags & BKMOO_FLAG_FUSED) && K <= kFusedMaxK) {
+  if (path == 2) {
     int64_t nmax = 0;
     for (int64_t b = 0; b < n_buckets; ++b)
       if (offsets[b + 1] - offsets[b] > nmax) nmax = offsets[b + 1] - offsets[b];
@@ -712,6 +738,15 @@ const char* bkmoo_status_string(int32_t status) {
 }
 
 int32_t bkmoo_version(void) { return kVersion; }
+
+int bkmoo_resolve_path(int32_t K, int32_t in_dtype, int32_t rule, const int64_t* offsets,
+                       int64_t n_buckets, uint32_t flags, int32_t* path) {
+  if (!path || K < 1 || K > kMaxK || !dtype_ok(in_dtype) || rule < BKMOO_MGDA ||
+      rule > BKMOO_MEAN || !offsets_ok(offsets, n_buckets))
+    return BKMOO_ERR_INVALID;
+  *path = choose_path(K, in_dtype, rule, offsets, n_buckets, flags);
+  return BKMOO_OK;
+}
 
 int bkmoo_selftest_fp64(int32_t op, const double* a, const double* b, double* out, int64_t n,
                         void* stream) {

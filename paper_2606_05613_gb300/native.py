@@ -31,6 +31,7 @@ BKMOO_F32, BKMOO_BF16 = 0, 1
 BKMOO_FLAG_CLOSED_FORM_K2 = 0x1
 BKMOO_FLAG_POLISH = 0x2
 BKMOO_FLAG_FUSED = 0x4
+BKMOO_FLAG_THREE_PASS = 0x8
 BKMOO_FLAG_TEST_WITHHOLD = 0x100
 BKMOO_NOALLOC_SCRATCH_BYTES = 32 << 20
 BKMOO_NOALLOC_MAX_BUCKETS = 4096
@@ -103,6 +104,9 @@ def load():
         lib.bkmoo_status_string.argtypes = [i32]
         lib.bkmoo_version.restype = i32
         lib.bkmoo_version.argtypes = []
+        lib.bkmoo_resolve_path.restype = ctypes.c_int
+        lib.bkmoo_resolve_path.argtypes = [i32, i32, i32, vp, i64, ctypes.c_uint32,
+                                           ctypes.POINTER(ctypes.c_int32)]
         lib.bkmoo_selftest_fp64.restype = ctypes.c_int
         lib.bkmoo_selftest_fp64.argtypes = [i32, vp, vp, vp, i64, vp]
         _lib = lib
@@ -289,6 +293,18 @@ def bkmoo_status_string(code: int) -> str:
 
 def bkmoo_version() -> int:
     return int(load().bkmoo_version())
+
+
+def bkmoo_resolve_path(K: int, in_dtype: int, rule, offsets, flags: int) -> int:
+    """0: three launches; 1: cluster-per-bucket fused kernel; 2:
+    grid-synchronised fused kernel (the path bkmoo_resolve takes)."""
+    if isinstance(rule, str):
+        rule = RULES[rule]
+    off = _offsets_array(offsets)
+    out = ctypes.c_int32(-1)
+    _check(load().bkmoo_resolve_path(K, in_dtype, rule, off.ctypes.data, len(off) - 1, flags,
+                                     ctypes.byref(out)), "bkmoo_resolve_path")
+    return int(out.value)
 
 
 def bkmoo_selftest_fp64(op: int, a, b, out, stream=None):

@@ -314,3 +314,51 @@ def test_selftest_fp64_rejects_bad_arguments_without_launch():
     assert lib.bkmoo_selftest_fp64(1, p[0], None, p[2], -1, None) == bk.BKMOO_ERR_INVALID
     assert lib.bkmoo_selftest_fp64(1, p[0], None, p[2], 0, None) == bk.BKMOO_OK
     del keep
+
+
+def test_resolve_path_choice():
+    """The per-plan path rule (measured on GB300): the cluster-per-bucket
+    fused kernel for K = 4 with 2-8 MiB (fp32) or 4-8 MiB (bf16) buckets and
+    a rule other than CAGrad; the three launches otherwise; the flags force
+    either path."""
+    F32, BF16 = bk.BKMOO_F32, bk.BKMOO_BF16
+    MiB = inputs.MiB
+
+    def plan(n, bucket_bytes, eb):
+        return bk.bkmoo_plan([n], eb, bucket_bytes)
+
+    sweep4 = plan(10**9, 4 * MiB, 4)
+    assert bk.bkmoo_resolve_path(4, F32, "mgda", sweep4, 0) == 1
+    assert bk.bkmoo_resolve_path(4, F32, "pcgrad", sweep4, 0) == 1
+    assert bk.bkmoo_resolve_path(4, F32, "mean", sweep4, 0) == 1
+    assert bk.bkmoo_resolve_path(4, F32, "cagrad", sweep4, 0) == 0
+    assert bk.bkmoo_resolve_path(2, F32, "mgda", sweep4, 0) == 0
+    assert bk.bkmoo_resolve_path(8, F32, "mgda", sweep4, 0) == 0
+    assert bk.bkmoo_resolve_path(4, F32, "mgda", plan(10**9, MiB, 4), 0) == 0
+    assert bk.bkmoo_resolve_path(4, F32, "mgda", plan(10**9, 2 * MiB, 4), 0) == 1
+    assert bk.bkmoo_resolve_path(4, F32, "mgda", plan(10**9, 16 * MiB, 4), 0) == 0
+    assert bk.bkmoo_resolve_path(4, BF16, "mgda", plan(10**9, 2 * MiB, 2), 0) == 0
+    assert bk.bkmoo_resolve_path(4, BF16, "mgda", plan(10**9, 4 * MiB, 2), 0) == 1
+    # the benchmark workloads keep the three launches
+    for sizes, eb, K, dt in [(inputs.qwen3_8b_sizes(), 2, 4, BF16),
+                             (inputs.gpt2_small_sizes(), 4, 4, F32),
+                             (inputs.llama32_1b_sizes(), 2, 8, BF16)]:
+        off = bk.bkmoo_plan(sizes, eb, 25 * MiB)
+        assert bk.bkmoo_resolve_path(K, dt, "mgda", off, 0) == 0
+    # one bucket in range and a third of the elements in small buckets: not
+    # chosen; with the small buckets under a tenth of the elements: chosen
+    mixed = np.array([0, 2 * 2**20] + [2 * 2**20 + 10000 * (i + 1) for i in range(100)],
+                     dtype=np.int64)
+    assert bk.bkmoo_resolve_path(4, F32, "mgda", mixed, 0) == 0
+    mostly = np.array([0, 2 * 2**20] + [2 * 2**20 + 1000 * (i + 1) for i in range(100)],
+                      dtype=np.int64)
+    assert bk.bkmoo_resolve_path(4, F32, "mgda", mostly, 0) == 1
+    # flags
+    assert bk.bkmoo_resolve_path(4, F32, "mgda", sweep4, bk.BKMOO_FLAG_THREE_PASS) == 0
+    assert bk.bkmoo_resolve_path(2, F32, "mgda", sweep4, bk.BKMOO_FLAG_FUSED) == 1
+    assert bk.bkmoo_resolve_path(8, F32, "mgda", sweep4, bk.BKMOO_FLAG_FUSED) == 2
+    assert bk.bkmoo_resolve_path(16, F32, "mgda", sweep4, bk.BKMOO_FLAG_FUSED) == 0
+    assert bk.bkmoo_resolve_path(
+        4, F32, "mgda", sweep4, bk.BKMOO_FLAG_FUSED | bk.BKMOO_FLAG_TEST_WITHHOLD) == 2
+    with pytest.raises(bk.BkmooError):
+        bk.bkmoo_resolve_path(0, F32, "mgda", sweep4, 0)
