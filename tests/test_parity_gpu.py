@@ -384,6 +384,34 @@ def test_fused_deterministic_and_matches_three_pass():
     assert np.linalg.norm(df - d3) <= 1e-5 * np.linalg.norm(d3)
 
 
+@pytest.mark.parametrize("K", [2, 4, 8])
+def test_fused_in_place_equals_out_of_place(K):
+    """In place (the direction written over the first gradient) the fused
+    kernels give the bit-identical result: every output position is read,
+    through its thread's own prefetch, by the thread that writes it, after
+    every Gram read of the bucket."""
+    w = _workload(K, "bf16", RAGGED * 2, 180000, seed=30 + K)
+    off, hv, out1, beta1, _, _ = _run(w, "mgda", "bf16", params=_fused_params())
+    _, _, out2, beta2, _, _ = _run(w, "mgda", "bf16", params=_fused_params(), inplace=True)
+    np.testing.assert_array_equal(beta1, beta2)
+    assert torch.equal(out1, out2)
+
+
+def test_per_plan_path_runs_the_fused_kernel_where_chosen():
+    """A plan for which bkmoo_resolve_path picks the cluster kernel (K = 4,
+    4 MiB fp32 buckets) resolves by it by default: the result is the one of
+    the forced fused path, bit for bit, and matches the oracle."""
+    K = 4
+    w = _workload(K, "f32", [3 * (1 << 20) + 12345], 1 << 20, seed=91)
+    off = bk.bkmoo_plan(w.param_sizes, 4, w.bucket_bytes)
+    assert bk.bkmoo_resolve_path(K, bk.BKMOO_F32, "mgda", off, 0) == 1
+    _, hv, out_auto, beta_auto, st, _ = _run(w, "mgda", "f32")
+    _, _, out_f, beta_f, _, _ = _run(w, "mgda", "f32", params=_fused_params())
+    np.testing.assert_array_equal(beta_auto, beta_f)
+    assert torch.equal(out_auto, out_f)
+    _check_against_oracle(w, "mgda", off, hv, out_auto, beta_auto, st, "f32")
+
+
 def test_fused_workspace_mismatch_is_detected():
     w = _workload(2, "f32", [40000, 40000], 40000, seed=6)
     off = bk.bkmoo_plan(w.param_sizes, w.elem_bytes, w.bucket_bytes)
