@@ -534,7 +534,10 @@ def main():
         "vs_baseline": None, "dtype": "f32" if w.dtype == "f32" else "bf16",
         "data": "synthetic",
         "config": dict(base_config(w, off, a.rule),
-                       l2="inputs (%.1f GB) >> L2, no flush" % (grad_bytes / GB),
+                       l2=("inputs (%.1f GB) >> L2, no flush" % (grad_bytes / GB)
+                           if grad_bytes > 4 * 126e6 else
+                           "inputs (%.3f GB) fit in L2 and are not flushed: L2-resident "
+                           "timing" % (grad_bytes / GB)),
                        parallelism="replicas" if world > 1 else "1 GPU",
                        path=({1: "fused: one launch, a thread-block cluster per bucket, "
                                     "combination re-reads each bucket from L2",

@@ -223,10 +223,14 @@ int choose_path(int32_t K, int32_t dt, int32_t rule, const int64_t* off, int64_t
     }
     return K <= kFusedMaxK ? 2 : 0;
   }
-  // measured on GB300: the cluster kernel is faster only for K = 4 with
-  // mid-sized buckets (MGDA 4.69 vs 5.07 ms at 2 MiB fp32, 4.83 vs 5.01 ms at
-  // 4 MiB bf16; MEAN and PCGrad more, CAGrad slower)
-  if (K != 4 || rule == BKMOO_CAGRAD || B < 1) return 0;
+  // measured on GB300: the cluster kernel is faster for tiny plans, where
+  // one launch instead of three is what counts (K = 2, 4 buckets of 1 MiB:
+  // 29.6 vs 33.4 us; 8 buckets: 30.2 vs 33.7 us; K = 4 ties), and for K = 4
+  // with mid-sized buckets (MGDA 4.69 vs 5.07 ms at 2 MiB fp32, 4.83 vs
+  // 5.01 ms at 4 MiB bf16; MEAN and PCGrad more, CAGrad slower)
+  if (B < 1) return 0;
+  if (K <= 2 && B <= 8 && off[B] <= ((int64_t)1 << 22)) return 1;
+  if (K != 4 || rule == BKMOO_CAGRAD) return 0;
   int64_t smax = 0;
   for (int64_t b = 0; b < B; ++b) smax = off[b + 1] - off[b] > smax ? off[b + 1] - off[b] : smax;
   const double bytes = (double)smax * elem_bytes(dt), mib = 1024.0 * 1024.0;

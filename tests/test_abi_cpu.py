@@ -339,7 +339,12 @@ def test_resolve_path_choice():
     assert bk.bkmoo_resolve_path(4, F32, "mgda", plan(10**9, 16 * MiB, 4), 0) == 0
     assert bk.bkmoo_resolve_path(4, BF16, "mgda", plan(10**9, 2 * MiB, 2), 0) == 0
     assert bk.bkmoo_resolve_path(4, BF16, "mgda", plan(10**9, 4 * MiB, 2), 0) == 1
-    # the benchmark workloads keep the three launches
+    # tiny plans: one launch (K <= 2, at most 8 buckets and 4 Mi elements)
+    assert bk.bkmoo_resolve_path(2, F32, "mgda", plan(1 << 20, MiB, 4), 0) == 1
+    assert bk.bkmoo_resolve_path(2, F32, "cagrad", plan(1 << 21, MiB, 4), 0) == 1
+    assert bk.bkmoo_resolve_path(2, F32, "mgda", plan(1 << 23, MiB, 4), 0) == 0
+    assert bk.bkmoo_resolve_path(4, F32, "mgda", plan(1 << 20, MiB, 4), 0) == 0
+    # the benchmark's model workloads keep the three launches
     for sizes, eb, K, dt in [(inputs.qwen3_8b_sizes(), 2, 4, BF16),
                              (inputs.gpt2_small_sizes(), 4, 4, F32),
                              (inputs.llama32_1b_sizes(), 2, 8, BF16)]:

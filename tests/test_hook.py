@@ -89,10 +89,13 @@ def test_bucket_moo_in_backward_matches_resolve(rule, dt):
             gs = torch.autograd.grad(((m(xs[k]) - ys[k]) ** 2).mean(), params)
             ref.append(torch.cat([g.reshape(-1) for g in reversed(gs)]))
             assert torch.equal(moo.grads[k], ref[k]), k
-        # one resolve over the whole plan, same buffers
+        # one resolve over the whole plan, same buffers (the three-launch
+        # path, whose kernels the per-bucket resolve runs)
         out = torch.empty_like(d)
         beta = torch.empty(moo.layout.n_buckets, K, device="cuda")
-        moo.resolver.resolve(moo.grads, rule, out, out_weights=beta)
+        p3 = bk.bkmoo_default_params()
+        p3.flags |= bk.BKMOO_FLAG_THREE_PASS
+        moo.resolver.resolve(moo.grads, rule, out, params=p3, out_weights=beta)
         torch.cuda.synchronize()
         assert moo.resolver.status() == 0
         assert torch.equal(d, out)
@@ -134,7 +137,9 @@ def test_bucket_moo_unused_parameter_resolved_in_finish():
     d = moo.finish()
     torch.cuda.synchronize()
     out = torch.empty_like(d)
-    moo.resolver.resolve(moo.grads, "mgda", out)
+    p3 = bk.bkmoo_default_params()
+    p3.flags |= bk.BKMOO_FLAG_THREE_PASS
+    moo.resolver.resolve(moo.grads, "mgda", out, params=p3)
     torch.cuda.synchronize()
     assert torch.equal(d, out)
     assert torch.count_nonzero(extra.grad).item() == 0

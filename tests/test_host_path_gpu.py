@@ -30,11 +30,14 @@ def _host_run(w, rule, out_dt, window_elems, pinned=True, inplace=False, params=
     grads = inputs.generate(w, off, DEV)
     B, N = len(off) - 1, int(off[-1])
     res = bk.Resolver(w.K, _tdt(w.dtype), off, DEV)
-    # device-resident reference run
+    # device-resident reference run on the three-launch path (the host path
+    # runs the same kernels window by window)
     out_d = torch.empty(N, dtype=_tdt(out_dt), device=DEV)
     beta_d = torch.empty(B, w.K, device=DEV)
     st_d = torch.empty(B, dtype=torch.int32, device=DEV)
-    res.resolve(grads, rule, out_d, params=params, out_weights=beta_d, out_status=st_d)
+    p3 = params if params is not None else bk.bkmoo_default_params()
+    p3.flags |= bk.BKMOO_FLAG_THREE_PASS
+    res.resolve(grads, rule, out_d, params=p3, out_weights=beta_d, out_status=st_d)
     # host run
     host = [torch.empty(N, dtype=_tdt(w.dtype), pin_memory=pinned) for _ in range(w.K)]
     for h, g in zip(host, grads):
