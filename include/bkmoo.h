@@ -86,7 +86,12 @@ typedef enum { BKMOO_F32 = 0, BKMOO_BF16 = 1 } bkmoo_dtype;
                                           slower for small buckets, large
                                           buckets and K = 8.  Results agree
                                           with the three-pass path to
-                                          rounding, not bit for bit.         */
+                                          rounding, not bit for bit.  The
+                                          groups kernel's L2 budget and
+                                          look-ahead can be overridden with
+                                          the environment variables
+                                          BKMOO_FUSED_L2_BUDGET (bytes) and
+                                          BKMOO_FUSED_LOOKAHEAD (buckets).   */
 #define BKMOO_FLAG_THREE_PASS 0x8u     /* always the three-launch path (Gram,
                                           solve, combination); without it and
                                           without BKMOO_FLAG_FUSED the path is

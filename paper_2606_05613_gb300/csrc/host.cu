@@ -217,10 +217,7 @@ int choose_path(int32_t K, int32_t dt, int32_t rule, const int64_t* off, int64_t
                 uint32_t flags) {
   if (flags & BKMOO_FLAG_THREE_PASS) return 0;
   if (flags & BKMOO_FLAG_FUSED) {
-    if (K <= kClusterMaxK && !(flags & BKMOO_FLAG_TEST_WITHHOLD)) {
-      const char* fk = std::getenv("BKMOO_FUSED_KERNEL");
-      if (!(fk && std::strcmp(fk, "groups") == 0)) return 1;
-    }
+    if (K <= kClusterMaxK && !(flags & BKMOO_FLAG_TEST_WITHHOLD)) return 1;
     return K <= kFusedMaxK ? 2 : 0;
   }
   // measured on GB300: the cluster kernel is faster for tiny plans, where
