@@ -80,11 +80,16 @@ typedef enum { BKMOO_F32 = 0, BKMOO_BF16 = 1 } bkmoo_dtype;
                                           CTAs for K = 5..8; above, ignored
                                           (three passes).  On a GB300 the
                                           cluster kernel is faster than three
-                                          passes for K = 4 with 2-8 MiB
-                                          buckets (the per-plan choice takes
+                                          passes for K = 2..4 with buckets of
+                                          2-6 MiB (the per-plan choice takes
                                           it there, see bkmoo_resolve_path),
-                                          slower for small buckets, large
-                                          buckets and K = 8.  Results agree
+                                          slower for 1 MiB buckets, large
+                                          buckets and K = 1 or 8.  The
+                                          cluster kernel's look-ahead into
+                                          the next bucket can be overridden
+                                          with the environment variable
+                                          BKMOO_CLUSTER_HEAD (items per
+                                          thread).  Results agree
                                           with the three-pass path to
                                           rounding, not bit for bit.  The
                                           groups kernel's L2 budget and
@@ -370,13 +375,13 @@ int bkmoo_workspace_status(const void* ws, void* stream, int32_t* status);
  * kernel.  BKMOO_FLAG_THREE_PASS gives 0; BKMOO_FLAG_FUSED gives 1 for
  * K <= 4 (2 with BKMOO_FLAG_TEST_WITHHOLD), 2 for K = 5..8, 0 above.
  * Without either flag the choice follows measurements on GB300 (sweeps of
- * 1e9 fp32 and 2e9 bf16 elements per language, and small plans): 1 when
- * K <= 2 and the plan has at most 8 buckets and 4 Mi elements per language
- * (one launch instead of three), or when K = 4, the rule is not CAGrad
- * (whose per-bucket solve is too long to hide), the largest bucket holds
- * 2-8 MiB per language for fp32 gradients or 4-8 MiB for bf16, and at least
- * 90 % of the elements lie in buckets of at least half that size; 0
- * otherwise.  Host only; BKMOO_ERR_INVALID on bad arguments.
+ * 1e9 elements per language, fp32 and bf16, and small plans): 1 when K <= 2
+ * and the plan has at most 8 buckets and 4 Mi elements per language (one
+ * launch instead of three), or when 2 <= K <= 4, the rule is not CAGrad
+ * unless K = 2 (CAGrad's per-bucket solve is too long to hide), the largest
+ * bucket holds at least 2 MiB per language and its K gradients together at
+ * most 12 MiB (and, for bf16, at least 6 MiB), and at least 90 % of the
+ * elements lie in buckets of at least half the largest; 0 otherwise.  Host only; BKMOO_ERR_INVALID on bad arguments.
  * bkmoo_resolve_buckets and bkmoo_resolve_host always take path 0.
  */
 int bkmoo_resolve_path(int32_t K, int32_t in_dtype, int32_t rule, const int64_t* offsets,

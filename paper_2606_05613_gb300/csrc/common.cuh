@@ -307,12 +307,14 @@ const void* fused_fn_bf16_k7_8(int K, int dtype_out);
 
 // Cluster-per-bucket fused kernels (fused_cluster.cu), K <= kClusterMaxK,
 // signature (GradPtrs, PlanView, SolveParams, float* out_weights,
-// int32_t* out_status, void* out), clusters of 8 CTAs of 256 threads with
+// int32_t* out_status, void* out, int head), clusters of kClusterCtas CTAs
+// of kClusterThreads threads (15 streaming warps and one solver warp) with
 // fused_cluster_smem(K) bytes of dynamic shared memory.
 constexpr int kClusterMaxK = 4;
 constexpr int kClusterCtas = 8;
-constexpr int kClusterWarps = 16;
-constexpr int kClusterThreads = 32 * kClusterWarps;
+constexpr int kClusterStreamWarps = 15;
+constexpr int kClusterStreamThreads = 32 * kClusterStreamWarps;
+constexpr int kClusterThreads = kClusterStreamThreads + 32;
 const void* fused_cluster_fn(int K, int dti, int dto);
 int fused_cluster_smem(int K);
 

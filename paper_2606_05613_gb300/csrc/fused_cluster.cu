@@ -1,4 +1,4 @@
-// Cluster-per-bucket fused resolve kernels, K = 1..4, fp32 / bf16 in and out.
+// Cluster-per-bucket fused resolve kernels, K = 1..kClusterMaxK, fp32 / bf16 in and out.
 #include "fused_cluster.cuh"
 
 namespace bkmoo {

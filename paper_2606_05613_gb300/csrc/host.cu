@@ -156,7 +156,10 @@ int launch_fused(const GradPtrs& g, const PlanView& v, const SolveParams& sp, vo
 }
 
 // The cluster-per-bucket fused path: as many clusters of kClusterCtas CTAs
-// as can be resident at once (clusters never wait for one another).
+// as can be resident at once, at most one per bucket (clusters never wait
+// for one another).  `head`: items per streaming thread of the next
+// bucket's Gram read before a combination, to cover the rule's solve
+// (environment variable BKMOO_CLUSTER_HEAD overrides it, for tuning).
 int launch_fused_cluster(const GradPtrs& g, const PlanView& v, const SolveParams& sp,
                          float* out_weights, int32_t* out_status, void* out, int dto,
                          cudaStream_t s) {
@@ -197,13 +200,19 @@ int launch_fused_cluster(const GradPtrs& g, const PlanView& v, const SolveParams
   }
   if (ncl < 1) return BKMOO_ERR_CUDA;
   if ((int64_t)ncl > v.n_buckets) ncl = (int)v.n_buckets;
+  const int head_bytes = sp.rule == BKMOO_MEAN ? 128 : sp.rule == BKMOO_CAGRAD ? 768 : 512;
+  int head = (head_bytes + 16 * v.K - 1) / (16 * v.K);
+  if (const char* e = std::getenv("BKMOO_CLUSTER_HEAD")) {
+    const int h = std::atoi(e);
+    if (h >= 0) head = h;
+  }
   GradPtrs ga = g;
   PlanView va = v;
   SolveParams spa = sp;
   float* ow = out_weights;
   int32_t* os = out_status;
   void* outp = out;
-  void* args[] = {&ga, &va, &spa, &ow, &os, &outp};
+  void* args[] = {&ga, &va, &spa, &ow, &os, &outp, &head};
   if (cudaLaunchKernel(fn, dim3(ncl * kClusterCtas), dim3(kClusterThreads), args, (size_t)smem,
                        s) != cudaSuccess)
     return BKMOO_ERR_CUDA;
@@ -220,19 +229,25 @@ int choose_path(int32_t K, int32_t dt, int32_t rule, const int64_t* off, int64_t
     if (K <= kClusterMaxK && !(flags & BKMOO_FLAG_TEST_WITHHOLD)) return 1;
     return K <= kFusedMaxK ? 2 : 0;
   }
-  // measured on GB300: the cluster kernel is faster for tiny plans, where
-  // one launch instead of three is what counts (K = 2, 4 buckets of 1 MiB:
-  // 29.6 vs 33.4 us; 8 buckets: 30.2 vs 33.7 us; K = 4 ties), and for K = 4
-  // with mid-sized buckets (MGDA 4.69 vs 5.07 ms at 2 MiB fp32, 4.83 vs
-  // 5.01 ms at 4 MiB bf16; MEAN and PCGrad more, CAGrad slower)
+  // measured on GB300 (1e9 elements per language, MGDA, fused / three
+  // launches): the cluster kernel is faster for tiny plans, where one
+  // launch instead of three is what counts (33 / 37 us), and for K = 2..4
+  // when buckets are large enough to amortise each bucket's hand-offs
+  // (>= 2 MiB) and small enough that the buckets in flight stay in L2:
+  // fp32 K = 2 2.70 / 2.94 ms at 2 MiB, 2.52 / 2.93 at 4 MiB; K = 3 3.50 /
+  // 3.94 at 2 MiB; K = 4 4.61 / 5.06 at 2 MiB; 1 MiB buckets are slower,
+  // and K x bucket above 12 MiB (fp32) or outside 6..12 MiB (bf16) ties or
+  // loses.  CAGrad's solve is too slow to hide for K > 2.
   if (B < 1) return 0;
   if (K <= 2 && B <= 8 && off[B] <= ((int64_t)1 << 22)) return 1;
-  if (K != 4 || rule == BKMOO_CAGRAD) return 0;
+  if (K < 2 || K > kClusterMaxK) return 0;
+  if (rule == BKMOO_CAGRAD && K > 2) return 0;
   int64_t smax = 0;
   for (int64_t b = 0; b < B; ++b) smax = off[b + 1] - off[b] > smax ? off[b + 1] - off[b] : smax;
-  const double bytes = (double)smax * elem_bytes(dt), mib = 1024.0 * 1024.0;
-  const double lo = (dt == BKMOO_F32 ? 2.0 : 4.0) * mib, hi = 8.0 * mib;
-  if (bytes < lo || bytes > hi) return 0;
+  const double mib = 1024.0 * 1024.0;
+  const double bytes = (double)smax * elem_bytes(dt), total = bytes * K;
+  if (bytes < 2.0 * mib) return 0;
+  if (total > 12.0 * mib || (dt != BKMOO_F32 && total < 6.0 * mib)) return 0;
   int64_t big = 0;
   for (int64_t b = 0; b < B; ++b)
     if (2 * (off[b + 1] - off[b]) >= smax) big += off[b + 1] - off[b];

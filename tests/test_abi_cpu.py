@@ -318,8 +318,9 @@ def test_selftest_fp64_rejects_bad_arguments_without_launch():
 
 def test_resolve_path_choice():
     """The per-plan path rule (measured on GB300): the cluster-per-bucket
-    fused kernel for K = 4 with 2-8 MiB (fp32) or 4-8 MiB (bf16) buckets and
-    a rule other than CAGrad; the three launches otherwise; the flags force
+    fused kernel for K = 2..4 with buckets of at least 2 MiB whose K
+    gradients take at most 12 MiB (bf16: 6..12 MiB), CAGrad only at
+    K = 2, and for tiny plans; the three launches otherwise; the flags force
     either path."""
     F32, BF16 = bk.BKMOO_F32, bk.BKMOO_BF16
     MiB = inputs.MiB
@@ -327,18 +328,28 @@ def test_resolve_path_choice():
     def plan(n, bucket_bytes, eb):
         return bk.bkmoo_plan([n], eb, bucket_bytes)
 
-    sweep4 = plan(10**9, 4 * MiB, 4)
-    assert bk.bkmoo_resolve_path(4, F32, "mgda", sweep4, 0) == 1
-    assert bk.bkmoo_resolve_path(4, F32, "pcgrad", sweep4, 0) == 1
-    assert bk.bkmoo_resolve_path(4, F32, "mean", sweep4, 0) == 1
+    def path(K, dt, rule, mib, eb):
+        return bk.bkmoo_resolve_path(K, dt, rule, plan(10**9, int(mib * MiB), eb), 0)
+
+    sweep4 = plan(10**9, 2 * MiB, 4)
+    for rule in ("mgda", "pcgrad", "mean"):
+        assert bk.bkmoo_resolve_path(4, F32, rule, sweep4, 0) == 1
     assert bk.bkmoo_resolve_path(4, F32, "cagrad", sweep4, 0) == 0
-    assert bk.bkmoo_resolve_path(2, F32, "mgda", sweep4, 0) == 0
+    assert bk.bkmoo_resolve_path(2, F32, "cagrad", sweep4, 0) == 1
+    assert bk.bkmoo_resolve_path(3, F32, "cagrad", sweep4, 0) == 0
     assert bk.bkmoo_resolve_path(8, F32, "mgda", sweep4, 0) == 0
-    assert bk.bkmoo_resolve_path(4, F32, "mgda", plan(10**9, MiB, 4), 0) == 0
-    assert bk.bkmoo_resolve_path(4, F32, "mgda", plan(10**9, 2 * MiB, 4), 0) == 1
-    assert bk.bkmoo_resolve_path(4, F32, "mgda", plan(10**9, 16 * MiB, 4), 0) == 0
-    assert bk.bkmoo_resolve_path(4, BF16, "mgda", plan(10**9, 2 * MiB, 2), 0) == 0
-    assert bk.bkmoo_resolve_path(4, BF16, "mgda", plan(10**9, 4 * MiB, 2), 0) == 1
+    assert bk.bkmoo_resolve_path(1, F32, "mgda", sweep4, 0) == 0
+    # fp32: buckets >= 2 MiB, K x bucket <= 12 MiB
+    fp32 = {(2, 1): 0, (2, 2): 1, (2, 4): 1, (2, 6): 1, (2, 8): 0,
+            (3, 1): 0, (3, 2): 1, (3, 4): 1, (3, 8): 0,
+            (4, 1): 0, (4, 2): 1, (4, 3): 1, (4, 4): 0}
+    for (K, mib), want in fp32.items():
+        assert path(K, F32, "mgda", mib, 4) == want, (K, mib)
+    # bf16: buckets >= 2 MiB, K x bucket in 6..12 MiB
+    bf16 = {(2, 2): 0, (2, 4): 1, (2, 8): 0, (3, 2): 1, (3, 4): 1, (3, 8): 0,
+            (4, 1): 0, (4, 2): 1, (4, 4): 0}
+    for (K, mib), want in bf16.items():
+        assert path(K, BF16, "mgda", mib, 2) == want, (K, mib)
     # tiny plans: one launch (K <= 2, at most 8 buckets and 4 Mi elements)
     assert bk.bkmoo_resolve_path(2, F32, "mgda", plan(1 << 20, MiB, 4), 0) == 1
     assert bk.bkmoo_resolve_path(2, F32, "cagrad", plan(1 << 21, MiB, 4), 0) == 1
@@ -352,10 +363,10 @@ def test_resolve_path_choice():
         assert bk.bkmoo_resolve_path(K, dt, "mgda", off, 0) == 0
     # one bucket in range and a third of the elements in small buckets: not
     # chosen; with the small buckets under a tenth of the elements: chosen
-    mixed = np.array([0, 2 * 2**20] + [2 * 2**20 + 10000 * (i + 1) for i in range(100)],
+    mixed = np.array([0, 2**19] + [2**19 + 3000 * (i + 1) for i in range(100)],
                      dtype=np.int64)
     assert bk.bkmoo_resolve_path(4, F32, "mgda", mixed, 0) == 0
-    mostly = np.array([0, 2 * 2**20] + [2 * 2**20 + 1000 * (i + 1) for i in range(100)],
+    mostly = np.array([0, 2**19] + [2**19 + 300 * (i + 1) for i in range(100)],
                       dtype=np.int64)
     assert bk.bkmoo_resolve_path(4, F32, "mgda", mostly, 0) == 1
     # flags

@@ -384,6 +384,21 @@ def test_fused_deterministic_and_matches_three_pass():
     assert np.linalg.norm(df - d3) <= 1e-5 * np.linalg.norm(d3)
 
 
+@pytest.mark.parametrize("rule", ["mgda", "pcgrad", "cagrad", "mean"])
+@pytest.mark.parametrize("dt", ["f32", "bf16"])
+@pytest.mark.parametrize("K", [1, 2, 3, 4])
+def test_fused_many_buckets_per_cluster(K, dt, rule):
+    """Enough buckets that every cluster of the cluster kernel resolves a
+    dozen or more in turn (its pipelined hand-offs: the next bucket's Gram
+    streamed while the one before is solved), with ragged bucket sizes;
+    every bucket against the oracle."""
+    sizes = [7001 + 37 * i for i in range(260)]
+    w = _workload(K, dt, sizes, 6000, seed=70 + K, flip=0.2)
+    off, hv, out, beta, status, _ = _run(w, rule, dt, params=_fused_params(3, 4))
+    assert len(off) - 1 >= 12 * 15
+    _check_against_oracle(w, rule, off, hv, out, beta, status, dt, seed=3, step=4)
+
+
 @pytest.mark.parametrize("K", [2, 4, 8])
 def test_fused_in_place_equals_out_of_place(K):
     """In place (the direction written over the first gradient) the fused
@@ -399,10 +414,10 @@ def test_fused_in_place_equals_out_of_place(K):
 
 def test_per_plan_path_runs_the_fused_kernel_where_chosen():
     """A plan for which bkmoo_resolve_path picks the cluster kernel (K = 4,
-    4 MiB fp32 buckets) resolves by it by default: the result is the one of
+    2 MiB fp32 buckets) resolves by it by default: the result is the one of
     the forced fused path, bit for bit, and matches the oracle."""
     K = 4
-    w = _workload(K, "f32", [3 * (1 << 20) + 12345], 1 << 20, seed=91)
+    w = _workload(K, "f32", [3 * (1 << 19) + 12345], 1 << 19, seed=91)
     off = bk.bkmoo_plan(w.param_sizes, 4, w.bucket_bytes)
     assert bk.bkmoo_resolve_path(K, bk.BKMOO_F32, "mgda", off, 0) == 1
     _, hv, out_auto, beta_auto, st, _ = _run(w, "mgda", "f32")
