@@ -765,6 +765,71 @@ __device__ void mgda_refine(const double* G, unsigned mask, const float (&Ainv)[
   for (int k = 0; k < K; ++k) alpha[k] *= corr;
 }
 
+// The same refinement step with its fp64 work spread over the warp, for
+// K <= 4 (every lane calls it; the winner lane `win` holds Ainv and z32).  On
+// this GPU an fp64 warp instruction costs tens of cycles whatever the number
+// of active lanes, so the serial form above spends most of a solve in its
+// ~60 of them: here lane l = 4 i + j forms the residual's term (i, j) of the
+// bordered system (row K: the simplex row), a two-level butterfly adds each
+// row, the winner applies its fp32 inverse, and lane k forms alpha_k.
+// Returns alpha_k on lane k < K, 0 on the other lanes.
+template <int K>
+__device__ double mgda_refine_warp(const double* G, unsigned mask, int win,
+                                   const float (&Ainv)[K + 1][K + 1], const float (&z32)[K + 1],
+                                   int lane) {
+  static_assert(K >= 1 && K <= 4, "rows of four lanes");
+  constexpr int N = K + 1;
+  float z[N];
+#pragma unroll
+  for (int c = 0; c < N; ++c) z[c] = __shfl_sync(0xffffffffu, z32[c], win);
+  const int i = lane >> 2, j = lane & 3;
+  float zi = 0.0f, zj = 0.0f;
+#pragma unroll
+  for (int c = 0; c < K; ++c) {
+    if (i == c) zi = z[c];
+    if (j == c) zj = z[c];
+  }
+  // term (i, j): G_ij z_j on the rows of G, z_j on the simplex row
+  const bool col_in = j < K && in_mask<K>(mask, j);
+  const double g = (i < K && j < K) ? G[i * K + j] : 1.0;
+  double term = col_in ? g * (double)zj : 0.0;
+  term += __shfl_xor_sync(0xffffffffu, term, 1);
+  term += __shfl_xor_sync(0xffffffffu, term, 2);
+  // residual of row i on its first lane: -(z_K + row) in S, -z_i outside,
+  // 1 - sum on the simplex row
+  double r;
+  if (i < K)
+    r = in_mask<K>(mask, i) ? -((double)z[K] + term) : -(double)zi;
+  else
+    r = 1.0 - term;
+  const float rf = (float)r;
+  float rr[N];
+#pragma unroll
+  for (int c = 0; c < N; ++c) rr[c] = __shfl_sync(0xffffffffu, rf, 4 * c);
+  // correction through the winner's fp32 inverse
+  float dk = 0.0f, zk = 0.0f;
+#pragma unroll
+  for (int c = 0; c < K; ++c) {
+    float t = 0.0f;
+#pragma unroll
+    for (int jj = 0; jj < N; ++jj) t = fmaf(Ainv[c][jj], rr[jj], t);
+    t = __shfl_sync(0xffffffffu, t, win);
+    if (lane == c) {
+      dk = t;
+      zk = z[c];
+    }
+  }
+  double a = 0.0;
+  if (lane < K) {
+    a = (double)zk + (double)dk;
+    a = (in_mask<K>(mask, lane) && a > 0.0) ? a : 0.0;
+  }
+  double s = a;
+  s += __shfl_xor_sync(0xffffffffu, s, 1);
+  s += __shfl_xor_sync(0xffffffffu, s, 2);
+  return a * (2.0 - s);  // 2 - s = 1 / s to first order, s = 1 + O(1e-16)
+}
+
 // Exact MGDA for 2 <= K <= 5.  False (beta untouched) if the optimality
 // check fails; the caller then takes the serial fp64 path.
 template <int K>
@@ -776,18 +841,30 @@ __device__ bool mgda_fast(const double* G, const float* Gf, int lane, double* be
   if (mask < (1u << K)) q = mgda_candidate32<K>(Gf, mask, Ainv, z);
   const int win = warp_argmin(q, lane);
   const unsigned wmask = (unsigned)win + 1u;
-  double alpha[K];
-  if (lane == win) mgda_refine<K>(G, wmask, Ainv, z, alpha);
-#pragma unroll
-  for (int k = 0; k < K; ++k) alpha[k] = __shfl_sync(0xffffffffu, alpha[k], win);
   if (!(__shfl_sync(0xffffffffu, q, win) < INFINITY)) return false;
+  double alpha[K];
+  float a32[K];
+  if constexpr (K <= 4) {
+    const double mine = mgda_refine_warp<K>(G, wmask, win, Ainv, z, lane);
+    const float mine32 = (float)mine;
+#pragma unroll
+    for (int k = 0; k < K; ++k) {
+      alpha[k] = __shfl_sync(0xffffffffu, mine, k);
+      a32[k] = __shfl_sync(0xffffffffu, mine32, k);
+    }
+  } else {
+    if (lane == win) mgda_refine<K>(G, wmask, Ainv, z, alpha);
+#pragma unroll
+    for (int k = 0; k < K; ++k) {
+      alpha[k] = __shfl_sync(0xffffffffu, alpha[k], win);
+      a32[k] = (float)alpha[k];
+    }
+  }
   // optimality: <g_k, d> >= ||d||^2 for every k (proof of Theorem 3.1); on
   // S it holds with equality by construction, off S it is checked in fp32
   // with a margin far above fp32 rounding, and in fp64 only when marginal
   {
-    float a32[K], v32[K], xx32 = 0.0f;
-#pragma unroll
-    for (int k = 0; k < K; ++k) a32[k] = (float)alpha[k];
+    float v32[K], xx32 = 0.0f;
 #pragma unroll
     for (int k = 0; k < K; ++k) {
       float t = 0.0f;
