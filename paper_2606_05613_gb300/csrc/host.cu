@@ -162,7 +162,7 @@ int launch_fused(const GradPtrs& g, const PlanView& v, const SolveParams& sp, vo
 // (environment variable BKMOO_CLUSTER_HEAD overrides it, for tuning).
 int launch_fused_cluster(const GradPtrs& g, const PlanView& v, const SolveParams& sp,
                          float* out_weights, int32_t* out_status, void* out, int dto,
-                         cudaStream_t s) {
+                         int64_t smax, cudaStream_t s) {
   if (cudaMemsetAsync(&v.hdr->status, 0, sizeof(int32_t), s) != cudaSuccess) return BKMOO_ERR_CUDA;
   if (v.n_buckets == 0) return BKMOO_OK;
   const void* fn = fused_cluster_fn(v.K, v.in_dtype, dto);
@@ -200,8 +200,15 @@ int launch_fused_cluster(const GradPtrs& g, const PlanView& v, const SolveParams
   }
   if (ncl < 1) return BKMOO_ERR_CUDA;
   if ((int64_t)ncl > v.n_buckets) ncl = (int)v.n_buckets;
-  const int head_bytes = sp.rule == BKMOO_MEAN ? 128 : sp.rule == BKMOO_CAGRAD ? 768 : 512;
-  int head = (head_bytes + 16 * v.K - 1) / (16 * v.K);
+  // look-ahead: 512 bytes of gradients per streaming thread (32 / K items),
+  // or the whole next bucket when it has at most 24 items per thread
+  // (measured best on GB300: K = 2 16 items, K = 3 11, K = 4 8-12 at 2 MiB
+  // fp32 buckets, the whole bucket at 1 MiB)
+  const int64_t eb = elem_bytes(v.in_dtype), epv = 16 / eb;
+  const int64_t items = (smax / epv / kClusterCtas + kClusterStreamThreads - 1) / kClusterStreamThreads;
+  int64_t h = items <= 24 ? items : 32 / v.K;
+  if (h < 2) h = 2;
+  int head = (int)h;
   if (const char* e = std::getenv("BKMOO_CLUSTER_HEAD")) {
     const int h = std::atoi(e);
     if (h >= 0) head = h;
@@ -231,13 +238,14 @@ int choose_path(int32_t K, int32_t dt, int32_t rule, const int64_t* off, int64_t
   }
   // measured on GB300 (1e9 elements per language, MGDA, fused / three
   // launches): the cluster kernel is faster for tiny plans, where one
-  // launch instead of three is what counts (33 / 37 us), and for K = 2..4
+  // launch instead of three is what counts (33 / 43 us), and for K = 2..4
   // when buckets are large enough to amortise each bucket's hand-offs
   // (>= 2 MiB) and small enough that the buckets in flight stay in L2:
-  // fp32 K = 2 2.70 / 2.94 ms at 2 MiB, 2.52 / 2.93 at 4 MiB; K = 3 3.50 /
-  // 3.94 at 2 MiB; K = 4 4.61 / 5.06 at 2 MiB; 1 MiB buckets are slower,
-  // and K x bucket above 12 MiB (fp32) or outside 6..12 MiB (bf16) ties or
-  // loses.  CAGrad's solve is too slow to hide for K > 2.
+  // fp32 K = 2 2.71 / 2.97 ms at 2 MiB, 2.50 / 2.95 at 4 MiB; K = 3 3.43 /
+  // 3.95 at 2 MiB; K = 4 4.59 / 5.07 at 2 MiB, 4.74 / 5.06 at 3 MiB; 1 MiB
+  // buckets are slower or tie, and K x bucket above 12 MiB (fp32) or
+  // outside 6..12 MiB (bf16) ties or loses.  CAGrad's solve is too slow to
+  // hide for K > 2.
   if (B < 1) return 0;
   if (K <= 2 && B <= 8 && off[B] <= ((int64_t)1 << 22)) return 1;
   if (K < 2 || K > kClusterMaxK) return 0;
@@ -530,17 +538,18 @@ int bkmoo_resolve(const void* const* grads, int32_t K, int32_t in_dtype, const i
   const SolveParams sp = solve_params(rule, prm);
   if (ev && cudaEventRecord(ev[0], s) != cudaSuccess) return BKMOO_ERR_CUDA;
   const int path = choose_path(K, in_dtype, rule, offsets, n_buckets, prm.flags);
+  int64_t nmax = 0;
+  if (path != 0)
+    for (int64_t b = 0; b < n_buckets; ++b)
+      if (offsets[b + 1] - offsets[b] > nmax) nmax = offsets[b + 1] - offsets[b];
   if (path == 1) {
-    r = launch_fused_cluster(g, v, sp, out_weights, out_status, out_dir, out_dtype, s);
+    r = launch_fused_cluster(g, v, sp, out_weights, out_status, out_dir, out_dtype, nmax, s);
     if (r != BKMOO_OK) return r;
     for (int i = 1; i < 4; ++i)
       if (ev && cudaEventRecord(ev[i], s) != cudaSuccess) return BKMOO_ERR_CUDA;
     return BKMOO_OK;
   }
   if (path == 2) {
-    int64_t nmax = 0;
-    for (int64_t b = 0; b < n_buckets; ++b)
-      if (offsets[b + 1] - offsets[b] > nmax) nmax = offsets[b + 1] - offsets[b];
     r = launch_fused(g, v, sp, ws, out_weights, out_status, out_dir, out_dtype,
                      (double)nmax * (K * elem_bytes(in_dtype) + elem_bytes(out_dtype)), s);
     if (r != BKMOO_OK) return r;
