@@ -377,10 +377,10 @@ int bkmoo_workspace_status(const void* ws, void* stream, int32_t* status);
  * Without either flag the choice follows measurements on GB300 (sweeps of
  * 1e9 elements per language, fp32 and bf16, and small plans): 1 when K <= 2
  * and the plan has at most 8 buckets and 4 Mi elements per language (one
- * launch instead of three), or when 2 <= K <= 4, the rule is not CAGrad
- * unless K = 2 (CAGrad's per-bucket solve is too long to hide), the largest
- * bucket holds at least 2 MiB per language and its K gradients together at
- * most 12 MiB (and, for bf16, at least 6 MiB), and at least 90 % of the
+ * launch instead of three), or when 2 <= K <= 4, the largest bucket holds at
+ * least 2 MiB per language and its K gradients together at most 12 MiB
+ * (and at least 6 MiB for bf16; for CAGrad, whose per-bucket solve is
+ * longer, fp32 only and at least 8 MiB), and at least 90 % of the
  * elements lie in buckets of at least half the largest; 0 otherwise.  Host only; BKMOO_ERR_INVALID on bad arguments.
  * bkmoo_resolve_buckets and bkmoo_resolve_host always take path 0.
  */

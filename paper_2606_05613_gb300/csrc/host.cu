@@ -244,18 +244,19 @@ int choose_path(int32_t K, int32_t dt, int32_t rule, const int64_t* off, int64_t
   // fp32 K = 2 2.71 / 2.97 ms at 2 MiB, 2.50 / 2.95 at 4 MiB; K = 3 3.43 /
   // 3.95 at 2 MiB; K = 4 4.59 / 5.07 at 2 MiB, 4.74 / 5.06 at 3 MiB; 1 MiB
   // buckets are slower or tie, and K x bucket above 12 MiB (fp32) or
-  // outside 6..12 MiB (bf16) ties or loses.  CAGrad's solve is too slow to
-  // hide for K > 2.
+  // outside 6..12 MiB (bf16) ties or loses.  CAGrad, whose solve takes
+  // 5.5-7 us, gains only from 8 MiB of fp32 gradients per bucket (K = 4
+  // 2 MiB 4.95 / 5.06, K = 2 4 MiB 2.73 / 2.93; K = 2 2 MiB and bf16 lose).
   if (B < 1) return 0;
   if (K <= 2 && B <= 8 && off[B] <= ((int64_t)1 << 22)) return 1;
   if (K < 2 || K > kClusterMaxK) return 0;
-  if (rule == BKMOO_CAGRAD && K > 2) return 0;
   int64_t smax = 0;
   for (int64_t b = 0; b < B; ++b) smax = off[b + 1] - off[b] > smax ? off[b + 1] - off[b] : smax;
   const double mib = 1024.0 * 1024.0;
   const double bytes = (double)smax * elem_bytes(dt), total = bytes * K;
   if (bytes < 2.0 * mib) return 0;
   if (total > 12.0 * mib || (dt != BKMOO_F32 && total < 6.0 * mib)) return 0;
+  if (rule == BKMOO_CAGRAD && (dt != BKMOO_F32 || total < 8.0 * mib)) return 0;
   int64_t big = 0;
   for (int64_t b = 0; b < B; ++b)
     if (2 * (off[b + 1] - off[b]) >= smax) big += off[b + 1] - off[b];

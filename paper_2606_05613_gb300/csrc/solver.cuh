@@ -1159,6 +1159,210 @@ __device__ bool cagrad_fast(const double* G, const float* Gf, double c, int lane
   return true;
 }
 
+// CAGrad for K <= 4 with the fp64 work spread over the warp (lane l = 4 i + j
+// holds entry (i, j) of G; every fp64 warp instruction costs tens of cycles
+// on this GPU however few lanes are active): the same candidates, one
+// refinement step of G_SS m = 1 and G_SS n = b with residuals in fp64, and
+// the same optimality check as cagrad_fast.  On S the weights are
+// w ~ (on + sqrt(D)) m - om n (lambda m - n with lambda = (on + sqrt(D)) / om,
+// times om), normalised by their fp64 sum: one division instead of two.
+template <int K>
+__device__ bool cagrad_fast_warp(const double* G, const float* Gf, double c, int lane,
+                                 double* beta_out) {
+  static_assert(K >= 1 && K <= 4, "rows of four lanes");
+  const int i = lane >> 2, j = lane & 3;
+  const double gij = (i < K && j < K) ? G[i * K + j] : 0.0;
+  // b_i = (G 1)_i / K on the lanes of row i, ||g0||^2 = 1^T G 1 / K^2
+  double row = gij;
+  row += __shfl_xor_sync(0xffffffffu, row, 1);
+  row += __shfl_xor_sync(0xffffffffu, row, 2);
+  double tot = j == 0 ? row : 0.0;
+  tot += __shfl_xor_sync(0xffffffffu, tot, 4);
+  tot += __shfl_xor_sync(0xffffffffu, tot, 8);
+  tot = __shfl_sync(0xffffffffu, tot, 0);
+  const double bi = row * (1.0 / K);
+  const float bif = (float)bi;
+  double b[K];
+  float bf[K];
+#pragma unroll
+  for (int k = 0; k < K; ++k) {
+    b[k] = __shfl_sync(0xffffffffu, bi, 4 * k);
+    bf[k] = __shfl_sync(0xffffffffu, bif, 4 * k);
+  }
+  const double g0sq = tot * (1.0 / ((double)K * K));
+  if (!(c > 0.0) || !(g0sq > 0.0)) {
+    if (lane < K) beta_out[lane] = 1.0 / K;
+    return true;
+  }
+  const double rho = c * sqrt_nr(g0sq);
+  float Ginv[K][K], w32[K];
+  const unsigned mask = (unsigned)lane + 1u;
+  float F = INFINITY;
+  if (mask < (1u << K)) F = cagrad_candidate32<K>(Gf, bf, (float)rho, mask, Ginv, w32);
+  const int win = warp_argmin(F, lane);
+  if (!(__shfl_sync(0xffffffffu, F, win) < INFINITY)) return false;
+  const unsigned wm = (unsigned)win + 1u;
+  const bool kin = lane < K && in_mask<K>(wm, lane);
+  double w = 0.0;  // w_k on lane k
+  if (__popc(wm) == 1) {
+    w = kin ? 1.0 : 0.0;
+  } else {
+    // m = Ginv 1_S and n = Ginv b_S from the winner (fp32), on every lane
+    float m[K], n[K];
+#pragma unroll
+    for (int ii = 0; ii < K; ++ii) {
+      float mi = 0.0f, ni = 0.0f;
+#pragma unroll
+      for (int jj = 0; jj < K; ++jj)
+        if (in_mask<K>(wm, jj)) {
+          mi += Ginv[ii][jj];
+          ni = fmaf(Ginv[ii][jj], bf[jj], ni);
+        }
+      m[ii] = __shfl_sync(0xffffffffu, mi, win);
+      n[ii] = __shfl_sync(0xffffffffu, ni, win);
+    }
+    float mj = 0.0f, nj = 0.0f, mi_ = 0.0f, ni_ = 0.0f;
+#pragma unroll
+    for (int cc = 0; cc < K; ++cc) {
+      if (j == cc) {
+        mj = m[cc];
+        nj = n[cc];
+      }
+      if (i == cc) {
+        mi_ = m[cc];
+        ni_ = n[cc];
+      }
+    }
+    // residuals of rows i in S (1 - (G m)_i, b_i - (G n)_i); -m_i, -n_i outside
+    const bool iin = i < K && in_mask<K>(wm, i);
+    const double g = (j < K && in_mask<K>(wm, j)) ? gij : 0.0;
+    double pm = g * (double)mj, pn = g * (double)nj;
+    pm += __shfl_xor_sync(0xffffffffu, pm, 1);
+    pn += __shfl_xor_sync(0xffffffffu, pn, 1);
+    pm += __shfl_xor_sync(0xffffffffu, pm, 2);
+    pn += __shfl_xor_sync(0xffffffffu, pn, 2);
+    const float rmf = (float)(iin ? 1.0 - pm : -(double)mi_);
+    const float rnf = (float)(iin ? bi - pn : -(double)ni_);
+    float rm[K], rn[K];
+#pragma unroll
+    for (int cc = 0; cc < K; ++cc) {
+      rm[cc] = __shfl_sync(0xffffffffu, rmf, 4 * cc);
+      rn[cc] = __shfl_sync(0xffffffffu, rnf, 4 * cc);
+    }
+    // the correction through the winner's inverse; m_k, n_k in fp64 on lane k
+    float mk = 0.0f, nk = 0.0f, dmk = 0.0f, dnk = 0.0f;
+#pragma unroll
+    for (int cc = 0; cc < K; ++cc) {
+      float dm = 0.0f, dn = 0.0f;
+#pragma unroll
+      for (int jj = 0; jj < K; ++jj) {
+        dm = fmaf(Ginv[cc][jj], rm[jj], dm);
+        dn = fmaf(Ginv[cc][jj], rn[jj], dn);
+      }
+      dm = __shfl_sync(0xffffffffu, dm, win);
+      dn = __shfl_sync(0xffffffffu, dn, win);
+      if (lane == cc) {
+        mk = m[cc];
+        nk = n[cc];
+        dmk = dm;
+        dnk = dn;
+      }
+    }
+    double bk = 0.0;
+#pragma unroll
+    for (int cc = 0; cc < K; ++cc)
+      if (lane == cc) bk = b[cc];
+    const double md = (double)mk + (double)dmk, nd = (double)nk + (double)dnk;
+    double om = kin ? md : 0.0, on = kin ? nd : 0.0, nb = kin ? nd * bk : 0.0;
+    om += __shfl_xor_sync(0xffffffffu, om, 1);
+    on += __shfl_xor_sync(0xffffffffu, on, 1);
+    nb += __shfl_xor_sync(0xffffffffu, nb, 1);
+    om += __shfl_xor_sync(0xffffffffu, om, 2);
+    on += __shfl_xor_sync(0xffffffffu, on, 2);
+    nb += __shfl_xor_sync(0xffffffffu, nb, 2);
+    om = __shfl_sync(0xffffffffu, om, 0);
+    on = __shfl_sync(0xffffffffu, on, 0);
+    nb = __shfl_sync(0xffffffffu, nb, 0);
+    const double D = on * on - om * (nb - rho * rho);
+    if (!(D > 0.0) || !(om > 0.0)) return false;
+    const double sd = sqrt_nr(D);
+    double u = kin ? fma(on + sd, md, -om * nd) : 0.0;
+    u = u > 0.0 ? u : 0.0;
+    double su = u;
+    su += __shfl_xor_sync(0xffffffffu, su, 1);
+    su += __shfl_xor_sync(0xffffffffu, su, 2);
+    su = __shfl_sync(0xffffffffu, su, 0);
+    if (!(su > 0.0)) return false;
+    w = div_nr(u, su);
+  }
+  // optimality of the dual: grad_k = b_k + rho (G w)_k / ||g_w|| >= w^T grad
+  // (equality on the support); fp32 with a margin, fp64 when marginal
+  const float wf_mine = (float)w;
+  float wf[K];
+#pragma unroll
+  for (int k = 0; k < K; ++k) wf[k] = __shfl_sync(0xffffffffu, wf_mine, k);
+  {
+    float v32[K], q32 = 0.0f;
+#pragma unroll
+    for (int k = 0; k < K; ++k) {
+      float t = 0.0f;
+#pragma unroll
+      for (int jj = 0; jj < K; ++jj) t = fmaf(Gf[k * K + jj], wf[jj], t);
+      v32[k] = t;
+      q32 = fmaf(wf[k], t, q32);
+    }
+    if (!(q32 > 1e-12f)) return false;
+    const float f32 = (float)rho / sqrtf(q32);
+    float lam32 = 0.0f, g32[K];
+#pragma unroll
+    for (int k = 0; k < K; ++k) {
+      g32[k] = fmaf(f32, v32[k], bf[k]);
+      lam32 = fmaf(wf[k], g32[k], lam32);
+    }
+    bool clear = true;
+#pragma unroll
+    for (int k = 0; k < K; ++k)
+      if (!in_mask<K>(wm, k) && !(g32[k] - lam32 >= 1e-5f)) clear = false;
+    if (!clear) {
+      double wd[K], v[K], qq = 0.0;
+#pragma unroll
+      for (int k = 0; k < K; ++k) wd[k] = __shfl_sync(0xffffffffu, w, k);
+#pragma unroll
+      for (int k = 0; k < K; ++k) {
+        double t = 0.0;
+#pragma unroll
+        for (int jj = 0; jj < K; ++jj) t = fma(G[k * K + jj], wd[jj], t);
+        v[k] = t;
+        qq = fma(wd[k], t, qq);
+      }
+      if (!(qq > 1e-24)) return false;
+      const double fd = div_nr(rho, sqrt_nr(qq));
+      double lam = 0.0, gmin = 1e300;
+#pragma unroll
+      for (int k = 0; k < K; ++k) {
+        const double gk = fma(fd, v[k], b[k]);
+        lam = fma(wd[k], gk, lam);
+        gmin = fmin(gmin, gk);
+      }
+      if (!(gmin >= lam - 1e-11)) return false;
+    }
+  }
+  // beta = 1/K + rho w / ||g_w||, ||g_w||^2 = w^T G w in fp64 (lane (i, j):
+  // w_i G_ij w_j, then a butterfly over the 16 lanes)
+  const double wi = __shfl_sync(0xffffffffu, w, i & 31);
+  const double wj = __shfl_sync(0xffffffffu, w, j);
+  double q = (i < K && j < K) ? gij * wi * wj : 0.0;
+  q += __shfl_xor_sync(0xffffffffu, q, 1);
+  q += __shfl_xor_sync(0xffffffffu, q, 2);
+  q += __shfl_xor_sync(0xffffffffu, q, 4);
+  q += __shfl_xor_sync(0xffffffffu, q, 8);
+  q = __shfl_sync(0xffffffffu, q, 0);
+  if (!(q > 1e-24)) return false;
+  const double f = div_nr(rho, sqrt_nr(q));
+  if (lane < K) beta_out[lane] = fma(f, w, 1.0 / K);
+  return true;
+}
+
 // PCGrad with one lane per task t < K (fp64): lane t runs the projections of
 // its running d_t in t's order; beta_j = sum_t C_tj by a fixed shuffle tree.
 template <int K>
@@ -1570,8 +1774,13 @@ __device__ bool solve_fast_k(int rule, const double* G, const float* Gf, const S
     if (K < 2 || (K == 2 && (p.flags & BKMOO_FLAG_CLOSED_FORM_K2))) return false;
     return mgda_fast<(K <= kEnumMaxK ? K : 2)>(G, Gf, lane, beta_out);
   }
-  if (rule == BKMOO_CAGRAD)
-    return cagrad_fast<(K <= kEnumMaxK ? K : 1)>(G, Gf, p.cagrad_c, lane, beta_out);
+  if (rule == BKMOO_CAGRAD) {
+    constexpr int KE = K <= kEnumMaxK ? K : 1;
+    if constexpr (KE <= 4)
+      return cagrad_fast_warp<KE>(G, Gf, p.cagrad_c, lane, beta_out);
+    else
+      return cagrad_fast<KE>(G, Gf, p.cagrad_c, lane, beta_out);
+  }
   return false;
 }
 

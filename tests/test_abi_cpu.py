@@ -319,9 +319,9 @@ def test_selftest_fp64_rejects_bad_arguments_without_launch():
 def test_resolve_path_choice():
     """The per-plan path rule (measured on GB300): the cluster-per-bucket
     fused kernel for K = 2..4 with buckets of at least 2 MiB whose K
-    gradients take at most 12 MiB (bf16: 6..12 MiB), CAGrad only at
-    K = 2, and for tiny plans; the three launches otherwise; the flags force
-    either path."""
+    gradients take at most 12 MiB (bf16: 6..12 MiB; CAGrad: fp32 and at
+    least 8 MiB), and for tiny plans; the three launches otherwise; the
+    flags force either path."""
     F32, BF16 = bk.BKMOO_F32, bk.BKMOO_BF16
     MiB = inputs.MiB
 
@@ -334,9 +334,13 @@ def test_resolve_path_choice():
     sweep4 = plan(10**9, 2 * MiB, 4)
     for rule in ("mgda", "pcgrad", "mean"):
         assert bk.bkmoo_resolve_path(4, F32, rule, sweep4, 0) == 1
-    assert bk.bkmoo_resolve_path(4, F32, "cagrad", sweep4, 0) == 0
-    assert bk.bkmoo_resolve_path(2, F32, "cagrad", sweep4, 0) == 1
+    # CAGrad: fp32 with at least 8 MiB of gradients per bucket
+    assert bk.bkmoo_resolve_path(4, F32, "cagrad", sweep4, 0) == 1
+    assert bk.bkmoo_resolve_path(2, F32, "cagrad", sweep4, 0) == 0
     assert bk.bkmoo_resolve_path(3, F32, "cagrad", sweep4, 0) == 0
+    assert path(2, F32, "cagrad", 4, 4) == 1
+    assert path(3, F32, "cagrad", 4, 4) == 1
+    assert path(4, BF16, "cagrad", 2, 2) == 0
     assert bk.bkmoo_resolve_path(8, F32, "mgda", sweep4, 0) == 0
     assert bk.bkmoo_resolve_path(1, F32, "mgda", sweep4, 0) == 0
     # fp32: buckets >= 2 MiB, K x bucket <= 12 MiB
