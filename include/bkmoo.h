@@ -112,6 +112,18 @@ typedef enum { BKMOO_F32 = 0, BKMOO_BF16 = 1 } bkmoo_dtype;
                                           ends with BKMOO_ERR_TIMEOUT in the
                                           workspace status word; the output
                                           is then undefined                 */
+#define BKMOO_FLAG_TEST_WITHHOLD_EXCHANGE 0x200u /* testing failure detection,
+                                          with BKMOO_FLAG_FUSED and K <= 4
+                                          only (the cluster kernel): CTA 0
+                                          of every cluster never hands its
+                                          partial Gram of the cluster's
+                                          first bucket to its peers, so the
+                                          peers' bounded exchange waits
+                                          (about 1 s) run out, every later
+                                          wait gives up at once, and the
+                                          call ends with BKMOO_ERR_TIMEOUT
+                                          in the workspace status word; the
+                                          output is then undefined          */
 
 typedef struct {
   int32_t max_iter; /* Frank-Wolfe iterations per bucket (MGDA, CAGrad)     */

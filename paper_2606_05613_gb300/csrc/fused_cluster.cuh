@@ -51,9 +51,10 @@
 // j + 1 only after passing barrier 2 for bucket j, and the solver arrives on
 // barrier 2 for bucket j + 1 only after passing barrier 1 for it.
 // Only the exchange waits poll; each gives up after about a second without
-// completion (BKMOO_ERR_TIMEOUT in the workspace status word, as soon as
-// any wait of the grid gave up), and the solver then carries on with what it
-// has so that every barrier is still reached.  A last cluster barrier keeps
+// completion, or at once when any wait of the grid already gave up
+// (BKMOO_ERR_TIMEOUT in the workspace status word), and the solver then
+// carries on with what it has so that every barrier is still reached; the
+// test flag BKMOO_FLAG_TEST_WITHHOLD_EXCHANGE exercises this path.  A last cluster barrier keeps
 // every CTA's shared memory alive until its peers are done with it.
 // Clusters never wait for one another, so they need not be co-resident.
 //
@@ -258,7 +259,10 @@ __device__ void cluster_solver_warp(const PlanView& v, const SolveParams& prm, f
     }
     __syncwarp();
     // 2. to every CTA of the cluster: lane r writes CTA r's copy and arrives
-    if (lane < W) {
+    // (BKMOO_FLAG_TEST_WITHHOLD_EXCHANGE: CTA 0 withholds its first one)
+    const bool withhold =
+        (prm.flags & BKMOO_FLAG_TEST_WITHHOLD_EXCHANGE) != 0u && rank == 0 && j == 0;
+    if (lane < W && !withhold) {
       double* dst = cluster.map_shared_rank(&xch[sl][rank][0], lane);
 #pragma unroll
       for (int p = 0; p < P; ++p) dst[p] = cta_sm[p];

@@ -33,6 +33,7 @@ BKMOO_FLAG_POLISH = 0x2
 BKMOO_FLAG_FUSED = 0x4
 BKMOO_FLAG_THREE_PASS = 0x8
 BKMOO_FLAG_TEST_WITHHOLD = 0x100
+BKMOO_FLAG_TEST_WITHHOLD_EXCHANGE = 0x200
 BKMOO_NOALLOC_SCRATCH_BYTES = 32 << 20
 BKMOO_NOALLOC_MAX_BUCKETS = 4096
 

@@ -380,5 +380,7 @@ def test_resolve_path_choice():
     assert bk.bkmoo_resolve_path(16, F32, "mgda", sweep4, bk.BKMOO_FLAG_FUSED) == 0
     assert bk.bkmoo_resolve_path(
         4, F32, "mgda", sweep4, bk.BKMOO_FLAG_FUSED | bk.BKMOO_FLAG_TEST_WITHHOLD) == 2
+    assert bk.bkmoo_resolve_path(
+        4, F32, "mgda", sweep4, bk.BKMOO_FLAG_FUSED | bk.BKMOO_FLAG_TEST_WITHHOLD_EXCHANGE) == 1
     with pytest.raises(bk.BkmooError):
         bk.bkmoo_resolve_path(0, F32, "mgda", sweep4, 0)

@@ -470,6 +470,37 @@ def test_fused_bounded_wait_reports_timeout():
     _check_against_oracle(w, "mgda", off, hv, out, beta.cpu().numpy(), status.cpu().numpy(), "bf16")
 
 
+def test_cluster_bounded_exchange_wait_reports_timeout():
+    """Failure detection in the cluster kernel without a fault: CTA 0 of
+    every cluster withholds its first bucket's partial (a hand-off that
+    never comes), each peer's exchange wait ends after its bound and every
+    later wait at once, the call reports BKMOO_ERR_TIMEOUT, and the context
+    stays usable: the next resolve succeeds and matches the oracle."""
+    import time
+    K = 4
+    sizes = [7001 + 37 * i for i in range(260)]
+    w = _workload(K, "f32", sizes, 6000, seed=29)
+    off = bk.bkmoo_plan(w.param_sizes, w.elem_bytes, w.bucket_bytes)
+    grads = inputs.generate(w, off, DEV)
+    res = bk.Resolver(K, torch.float32, off, DEV)
+    out = torch.empty(int(off[-1]), dtype=torch.float32, device=DEV)
+    p = _fused_params(flags=bk.bkmoo_default_params().flags
+                      | bk.BKMOO_FLAG_TEST_WITHHOLD_EXCHANGE)
+    assert bk.bkmoo_resolve_path(K, bk.BKMOO_F32, "mgda", off, p.flags) == 1
+    t0 = time.time()
+    res.resolve(grads, "mgda", out, params=p)
+    assert res.status() == bk.BKMOO_ERR_TIMEOUT
+    assert time.time() - t0 < 30.0
+    B = len(off) - 1
+    beta = torch.empty(B, K, device=DEV)
+    status = torch.empty(B, dtype=torch.int32, device=DEV)
+    res.resolve(grads, "mgda", out, params=_fused_params(), out_weights=beta, out_status=status)
+    torch.cuda.synchronize()
+    assert res.status() == 0
+    hv = [inputs.host_view(g) for g in grads]
+    _check_against_oracle(w, "mgda", off, hv, out, beta.cpu().numpy(), status.cpu().numpy(), "f32")
+
+
 @pytest.mark.parametrize("K", [2, 4, 8, 16])
 def test_conflict_statistics(K):
     """Figure 1 statistics from the GPU Gram against the oracle's (cosines to
