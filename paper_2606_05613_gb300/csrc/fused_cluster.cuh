@@ -68,8 +68,8 @@
 
 namespace bkmoo {
 
-// stages of the per-thread cp.async ring: 24 / K, i.e. 180 KiB of slots at
-// K = 1..4 but 3 (measured faster than 28 / K, the most that fits)
+// stages of the per-thread cp.async ring: 24 / K, i.e. 180 KiB of slots for
+// K = 1..4 (measured faster than 28 / K, the most that fits)
 __host__ __device__ constexpr int cluster_stages(int K) { return K >= 12 ? 2 : 24 / K; }
 __host__ __device__ constexpr int cluster_smem_bytes(int K) {
   return cluster_stages(K) * K * 16 * kClusterStreamThreads;
