@@ -8,10 +8,10 @@
 // fit on a 152-SM part; 9-CTA clusters cover more SMs but measured slower).
 // Cluster c resolves buckets c, c + n_clusters, ... in turn.  A bucket's
 // 16-byte vectors are cut into W equal pieces, one per CTA (the unaligned
-// head and tail elements go to the first and last piece).  A CTA has 15 streaming warps and one
-// solver warp; streaming thread t takes vectors t, t + 480, ... of the
-// piece, items 0, 1, ... in that order (a CTA step reads 7.5 KB of each
-// gradient contiguously).
+// head and tail elements go to the first and last piece).  A CTA has 15
+// streaming warps and one solver warp; streaming thread t takes vectors t,
+// t + 480, ... of the piece, items 0, 1, ... in that order (a CTA step reads
+// 7.5 KB of each gradient contiguously).
 //
 // Streaming warps walk a fixed schedule of segments,
 //   G(0), H(1), C(0), R(1), H(2), C(1), R(2), ..., C(J - 1),
@@ -54,9 +54,10 @@
 // completion, or at once when any wait of the grid already gave up
 // (BKMOO_ERR_TIMEOUT in the workspace status word), and the solver then
 // carries on with what it has so that every barrier is still reached; the
-// test flag BKMOO_FLAG_TEST_WITHHOLD_EXCHANGE exercises this path.  A last cluster barrier keeps
-// every CTA's shared memory alive until its peers are done with it.
-// Clusters never wait for one another, so they need not be co-resident.
+// test flag BKMOO_FLAG_TEST_WITHHOLD_EXCHANGE exercises this path.  A last
+// cluster barrier keeps every CTA's shared memory alive until its peers are
+// done with it.  Clusters never wait for one another, so they need not be
+// co-resident.
 //
 // Results are deterministic for a given cluster shape and count; the pieces
 // differ from the three-pass path's chunks, so the two agree to rounding.
@@ -87,7 +88,9 @@ __device__ __forceinline__ void mbar_init(uint64_t* bar, unsigned count) {
 // stores, local or remote, before the arrival).
 __device__ __forceinline__ void mbar_arrive_remote(uint64_t* bar, unsigned rank) {
   uint32_t remote;
-  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(remote) : "r"(smem_u32(bar)), "r"(rank));
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;"
+               : "=r"(remote)
+               : "r"(smem_u32(bar)), "r"(rank));
   asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(remote)
                : "memory");
 }
