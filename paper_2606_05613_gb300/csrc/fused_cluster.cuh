@@ -161,7 +161,7 @@ template <int T>
 __device__ __forceinline__ ClusterRange cluster_range(int kind, const Piece& pc, int t, int head) {
   const int64_t npc = pc.vhi - pc.vlo;
   const int n = (int)((npc + T - 1) / T);
-  const int h = head < n ? head : n;
+  const int h = head < 0 ? 0 : head < n ? head : n;
   ClusterRange r;
   r.i0 = kind == 3 ? h : 0;
   r.i1 = kind == 1 ? h : n;
