@@ -42,6 +42,27 @@ def test_library_exports_every_declared_symbol():
         assert hasattr(lib, n), n
 
 
+def test_binding_constants_match_the_header():
+    """Every enumerator and integer #define of include/bkmoo.h has the same
+    value in the binding (the binding restates them; nothing else ties the
+    two together)."""
+    import os
+    h = os.path.join(os.path.dirname(bk.LIB_PATH), "..", "include", "bkmoo.h")
+    src = re.sub(r"/\*.*?\*/", "", open(h).read(), flags=re.S)
+    consts = {}
+    for m in re.finditer(r"#define\s+(BKMOO_[A-Z0-9_]+)\s+\(?\s*(0x[0-9a-fA-F]+|\d+)u?"
+                         r"(?:\s*<<\s*(\d+)\s*\))?", src):
+        v = int(m.group(2), 0)
+        consts[m.group(1)] = v << int(m.group(3)) if m.group(3) else v
+    for body in re.findall(r"enum\s*\{(.*?)\}", src, flags=re.S):
+        for m in re.finditer(r"(BKMOO_[A-Z0-9_]+)\s*=\s*(\d+)", body):
+            consts[m.group(1)] = int(m.group(2))
+    assert len(consts) >= 20, sorted(consts)
+    for name, v in consts.items():
+        assert hasattr(bk, name), name
+        assert getattr(bk, name) == v, (name, getattr(bk, name), v)
+
+
 def test_version_and_status_strings():
     assert bk.bkmoo_version() == 200
     for code in range(8):
